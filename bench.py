@@ -1,0 +1,484 @@
+"""Benchmark of the mixed prefill+decode attention step (one JSON line).
+
+Default workload (low pressure, MBT 16384, Qwen2.5-3B attention geometry:
+16 q-heads, 2 kv-heads, head_dim 128, 36 layers): one 25,000-token prompt
+planned by the P-PAS planner into the chunks (16384, prefix 0) and
+(8616, prefix 16384).  One bench step = plan both iterations on the host,
+then for each iteration and each of the 36 layers append the chunk's keys and
+values and run the attention step.  Every layer has its own Q, K/V cache and
+output buffers, so the per-step inputs (about 7.7 GB) are far larger than L2.
+
+The high-pressure workload (MBT 2048: 4 prefill chunks of 512 with prefixes
+~U[0, 24576) batched with 8 decode rows of context ~U[25000, 25032), 36
+layers) is timed the same way and reported under ``mbt2k``.
+
+``--impl reference`` times the float64 CPU oracle instead, on a bounded
+sample of the same workload, extrapolated by causal pair count.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_15171_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "mixed prefill+decode attention step time (us) and % roofline at MBT 2k/16k"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# DRAM traffic of one prefill-kernel launch measured by ncu, keyed by the
+# sha256 of the kernel source it was measured on (reported only while the
+# source is unchanged).
+PREFILL_TRAFFIC = {}
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+def _src_hash(name):
+    with open(os.path.join(ROOT, "paper_2608_15171_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"ppas_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for ln in f:
+                parts = [x.strip() for x in ln.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": float(max(mx)), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- workloads
+class LayerSet:
+    """Per-layer device buffers of one workload (distinct for every layer)."""
+
+
+def _setup_low(torch, ppas, geo, dev, seed=0):
+    """Low-pressure workload: the planner's two iterations of a 25,000-token prompt."""
+    prompt = 25000
+    nb = wl.blocks_for(prompt) + 13
+    perm = wl.page_permutation(nb, seed)
+    W = LayerSet()
+    W.geo, W.nb, W.perm, W.prompt = geo, nb, perm, prompt
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    W.k_cache, W.v_cache, W.q, W.kn, W.vn, W.out = [], [], [], [], [], []
+    shapes = wl.low_pressure_steps()
+    W.shapes = shapes
+    for layer in range(geo.n_layers):
+        s = 1000 * layer + seed
+        W.k_cache.append(torch.zeros((nb, hk, 16, D), dtype=torch.bfloat16, device=dev))
+        W.v_cache.append(torch.zeros((nb, hk, 16, D), dtype=torch.bfloat16, device=dev))
+        W.q.append([wl.bf16_normal((sh.total_q, hq, D), s + 1 + i, dev) for i, sh in enumerate(shapes)])
+        W.kn.append([wl.bf16_normal((sh.total_q, hk, D), s + 11 + i, dev) for i, sh in enumerate(shapes)])
+        W.vn.append([wl.bf16_normal((sh.total_q, hk, D), s + 21 + i, dev) for i, sh in enumerate(shapes)])
+        W.out.append([torch.empty((sh.total_q, hq, D), dtype=torch.bfloat16, device=dev) for sh in shapes])
+    W.err = torch.zeros(1, dtype=torch.int32, device=dev)
+    # one set of plan buffers per iteration: a later iteration never
+    # overwrites host memory whose copy may still be queued
+    W.tables_dev = [torch.empty((1, 4096), dtype=torch.int32, device=dev) for _ in range(2)]
+    W.slots_dev = [torch.empty((32768,), dtype=torch.int32, device=dev) for _ in range(2)]
+    W.tables_pin = [torch.empty((1, 4096), dtype=torch.int32).pin_memory() for _ in range(2)]
+    W.slots_pin = [torch.empty((32768,), dtype=torch.int32).pin_memory() for _ in range(2)]
+    return W
+
+
+def _low_step(torch, ppas, W, stream, timers=None, host=None):
+    """One bench step of the low-pressure workload.  ``timers`` collects CUDA
+    events around each attention launch; ``host`` runs it end to end from
+    pinned host buffers (inputs copied in, outputs copied out)."""
+    geo = W.geo
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    sch = ppas.Scheduler(W.nb, W.perm, cap_rows=8, cap_blocks_per_seq=4096, cap_tokens=32768)
+    sch.add_requests([(0, W.prompt, 2)])
+    launches = 0
+    try:
+        for it in range(2):
+            st = sch.plan(0, 2, 16384, 2048)
+            n = st.total_tokens
+            width = st.block_table.shape[1]
+            W.tables_pin[it][0, :width].copy_(torch.from_numpy(st.block_table[0]))
+            W.slots_pin[it][:n].copy_(torch.from_numpy(st.slot_mapping))
+            W.tables_dev[it][0, :width].copy_(W.tables_pin[it][0, :width], non_blocking=True)
+            W.slots_dev[it][:n].copy_(W.slots_pin[it][:n], non_blocking=True)
+            tables = W.tables_dev[it][:, :width]
+            slots = W.slots_dev[it]
+            for layer in range(geo.n_layers):
+                q, kn, vn, out = W.q[layer][it], W.kn[layer][it], W.vn[layer][it], W.out[layer][it]
+                if host is not None:
+                    q.copy_(host["q"][it], non_blocking=True)
+                    kn.copy_(host["kn"][it], non_blocking=True)
+                    vn.copy_(host["vn"][it], non_blocking=True)
+                ppas.ppas_kv_append(kn, vn, slots, n, W.k_cache[layer], W.v_cache[layer], W.nb, hk, D,
+                                    W.err, stream)
+                if timers is not None:
+                    e0 = torch.cuda.Event(enable_timing=True)
+                    e0.record(stream)
+                ppas.ppas_attention_step(q, W.k_cache[layer], W.v_cache[layer], W.nb, tables, width, st.q_len,
+                                         st.ctx_len, hq, hk, D, geo.scale, out, False, None, 0, W.err, stream)
+                if timers is not None:
+                    e1 = torch.cuda.Event(enable_timing=True)
+                    e1.record(stream)
+                    timers.append((it, e0, e1))
+                if host is not None:
+                    host["out"][it].copy_(out, non_blocking=True)
+                launches += 2
+    finally:
+        sch.close()
+    return launches
+
+
+def _setup_high(torch, ppas, geo, dev, seed=0):
+    """High-pressure workload: literal step, contexts pre-filled into pages."""
+    shape = wl.high_pressure_step(seed)
+    W = LayerSet()
+    W.geo, W.shape = geo, shape
+    need = sum(wl.blocks_for(c) for c in shape.ctx_lens)
+    W.nb = need + 13
+    perm = wl.page_permutation(W.nb, seed + 7)
+    tables_np = wl.literal_tables(shape, perm)
+    W.width = tables_np.shape[1]
+    W.tables = torch.from_numpy(tables_np).to(dev)
+    slots = []
+    for s, (q, c) in enumerate(zip(shape.q_lens, shape.ctx_lens)):
+        pos = np.arange(c - q, c)
+        slots.append(tables_np[s][pos // 16] * 16 + pos % 16)
+    W.slots = torch.from_numpy(np.concatenate(slots).astype(np.int32)).to(dev)
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    T = shape.total_q
+    W.k_cache, W.v_cache, W.q, W.kn, W.vn, W.out = [], [], [], [], [], []
+    for layer in range(geo.n_layers):
+        s = 1000 * layer + seed + 500
+        W.k_cache.append(wl.bf16_normal((W.nb, hk, 16, D), s + 1, dev))
+        W.v_cache.append(wl.bf16_normal((W.nb, hk, 16, D), s + 2, dev))
+        W.q.append(wl.bf16_normal((T, hq, D), s + 3, dev))
+        W.kn.append(wl.bf16_normal((T, hk, D), s + 4, dev))
+        W.vn.append(wl.bf16_normal((T, hk, D), s + 5, dev))
+        W.out.append(torch.empty((T, hq, D), dtype=torch.bfloat16, device=dev))
+    W.ws_bytes = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, hq, hk)
+    W.ws = torch.empty(max(W.ws_bytes, 256), dtype=torch.uint8, device=dev)
+    W.err = torch.zeros(1, dtype=torch.int32, device=dev)
+    return W
+
+
+def _high_step(torch, ppas, W, stream, timers=None):
+    geo, sh = W.geo, W.shape
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    launches = 0
+    for layer in range(geo.n_layers):
+        ppas.ppas_kv_append(W.kn[layer], W.vn[layer], W.slots, sh.total_q, W.k_cache[layer], W.v_cache[layer],
+                            W.nb, hk, D, W.err, stream)
+        if timers is not None:
+            e0 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        ppas.ppas_attention_step(W.q[layer], W.k_cache[layer], W.v_cache[layer], W.nb, W.tables, W.width,
+                                 sh.q_lens, sh.ctx_lens, hq, hk, D, geo.scale, W.out[layer], False, W.ws, W.ws_bytes,
+                                 W.err, stream)
+        if timers is not None:
+            e1 = torch.cuda.Event(enable_timing=True)
+            e1.record(stream)
+            timers.append((0, e0, e1))
+        launches += 1 + 1 + (1 if any(q == 1 for q in sh.q_lens) else 0)
+    return launches
+
+
+def _roofline_time_us(shape, geo, peaks, sustained=True):
+    tf = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"] * 1e12
+    bw = peaks["hbm_gbs"] * 1e9
+    return max(wl.step_flops(shape, geo) / tf, wl.step_bytes(shape, geo) / bw) * 1e6
+
+
+def _timed(torch, dist, fn, steps, warmup, stream, rank, sample_clocks):
+    for _ in range(warmup):
+        fn(None)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    sampler = ClockSampler(torch.cuda.current_device()) if sample_clocks else None
+    if sampler:
+        sampler.start()
+        time.sleep(0.3)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    timers = []
+    launches = 0
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        launches += fn(timers)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    if dist is not None:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    clocks = sampler.stop() if sampler else None
+    return ms, timers, launches, clocks
+
+
+def run_ours(args, rank, world, dist):
+    import torch
+    from paper_2608_15171_gb300 import ppas
+
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream()
+    peaks, peaks_kind = _peaks()
+    geo = wl.QWEN25_3B
+
+    # ---- low pressure (MBT 16k): the headline step
+    W = _setup_low(torch, ppas, geo, dev)
+    ms, timers, launches, clocks = _timed(
+        torch, dist, lambda tm: _low_step(torch, ppas, W, stream, tm), args.steps, args.warmup, stream, rank, True)
+    assert W.err.item() == 0, f"device error flag {W.err.item()}"
+    per_launch = [(it, a.elapsed_time(b)) for it, a, b in timers]
+    shapes = W.shapes
+    flops_step = sum(wl.step_flops(sh, geo) for sh in shapes) * geo.n_layers
+    attn_ms = sum(t for _, t in per_launch) / args.steps
+    attn_flops_per_launch = flops_step / (2 * geo.n_layers)
+    avg_launch_ms = attn_ms / (2 * geo.n_layers)
+    achieved = attn_flops_per_launch / (avg_launch_ms * 1e-3) / 1e12
+    peak = peaks["bf16_tflops_sustained"]
+    roof_step_us = sum(_roofline_time_us(sh, geo, peaks) for sh in shapes) * geo.n_layers
+    step_us = ms * 1e3 / args.steps
+    traffic = PREFILL_TRAFFIC.get(_src_hash("attn_prefill.cu"))
+
+    # ---- end to end from pinned host buffers (inputs in, outputs out every layer)
+    host = {"q": [W.q[0][i].cpu().pin_memory() for i in range(2)],
+            "kn": [W.kn[0][i].cpu().pin_memory() for i in range(2)],
+            "vn": [W.vn[0][i].cpu().pin_memory() for i in range(2)],
+            "out": [torch.empty_like(W.out[0][i], device="cpu").pin_memory() for i in range(2)]}
+    e2e_steps = max(1, min(args.steps, 3))
+    ms_e2e, _, _, _ = _timed(torch, dist, lambda tm: _low_step(torch, ppas, W, stream, None, host), e2e_steps, 1,
+                             stream, rank, False)
+    h2d = sum((host["q"][i].nbytes + host["kn"][i].nbytes + host["vn"][i].nbytes) for i in range(2)) * geo.n_layers
+    d2h = sum(host["out"][i].nbytes for i in range(2)) * geo.n_layers
+    e2e = {"value": round(ms_e2e * 1e3 / e2e_steps, 1), "unit": "us",
+           "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+    del host
+    cpu_w = {"k": W.k_cache[0], "v": W.v_cache[0]}
+    W_low = W
+
+    # ---- high pressure (MBT 2k with 8 decodes)
+    H = _setup_high(torch, ppas, geo, dev)
+    ms_h, timers_h, launches_h, clocks_h = _timed(
+        torch, dist, lambda tm: _high_step(torch, ppas, H, stream, tm), args.steps, args.warmup, stream, rank, False)
+    assert H.err.item() == 0, f"device error flag {H.err.item()}"
+    hs_us = ms_h * 1e3 / args.steps
+    roof_h_us = _roofline_time_us(H.shape, geo, peaks) * geo.n_layers
+    attn_h_ms = sum(a.elapsed_time(b) for _, a, b in timers_h) / args.steps
+    mbt2k = {
+        "workload": "MBT 2048: 4x512 chunks, prefixes ~U[0,24576) + 8 decodes ctx ~U[25000,25032), 36 layers",
+        "q_lens": H.shape.q_lens, "ctx_lens": H.shape.ctx_lens,
+        "step_us": round(hs_us, 1), "attention_us_per_layer": round(attn_h_ms * 1e3 / geo.n_layers, 2),
+        "roofline_us": round(roof_h_us, 1), "frac": round(roof_h_us / hs_us, 4),
+        "frac_attention_only": round(roof_h_us / (attn_h_ms * 1e3), 4),
+        "tflops": round(wl.step_flops(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e12, 1),
+        "hbm_gbs": round(wl.step_bytes(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e9, 1)}
+    del H
+
+    line = {
+        "metric": METRIC, "value": round(step_us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "MBT 16384 low pressure: 25,000-token prompt planned into chunks (16384, p=0) and "
+                               "(8616, p=16384); Qwen2.5-3B attention geometry 16q/2kv/d128, 36 layers; "
+                               "plan + kv append + attention per layer",
+                   "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (distinct buffers per layer)",
+                   "step": "2 scheduler iterations x 36 layers"},
+        "roofline": {"bound": "tensor", "kernel": "prefill_attn_kernel", "achieved": round(achieved, 1),
+                     "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+                     "peak_kind": f"{peaks_kind} sustained bf16", "traffic": traffic,
+                     "avg_launch_us": round(avg_launch_ms * 1e3, 1),
+                     "flops_per_launch": attn_flops_per_launch},
+        "step_roofline": {"roofline_us": round(roof_step_us, 1), "frac": round(roof_step_us / step_us, 4),
+                          "frac_vs_burst_peak": round(
+                              sum(_roofline_time_us(sh, geo, peaks, False) for sh in shapes) * geo.n_layers
+                              / step_us, 4)},
+        "per_iteration_us": {
+            f"q={sh.q_lens[0]},p={sh.ctx_lens[0] - sh.q_lens[0]}": round(
+                sum(t for it, t in per_launch if it == i) * 1e3 / args.steps / geo.n_layers, 1)
+            for i, sh in enumerate(shapes)},
+        "mbt2k": mbt2k,
+        "e2e": e2e,
+        "gpu_launches": launches // args.steps * args.steps,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(W_low, cpu_w, torch, args)
+    return line
+
+
+def _oracle_sample(kc, vc, table, geo, rows, workers):
+    """Oracle on the last ``rows`` query tokens of the first 16384-token chunk
+    (all 16 heads); returns (seconds, causal pairs per head)."""
+    from oracle import attention as oa
+    L = 16384
+    q = wl.bf16_normal((rows, geo.n_q_heads, geo.head_dim), 77, "cpu").to(torch_float64())
+    t0 = time.perf_counter()
+    oa.paged_attention(q.numpy(), kc, vc, table, [rows], [L], geo.scale, workers=workers)
+    dt = time.perf_counter() - t0
+    p = L - rows
+    return dt, rows * p + rows * (rows + 1) // 2
+
+
+def torch_float64():
+    import torch
+    return torch.float64
+
+
+def _workload_pairs(geo):
+    return sum(wl.step_pairs(sh) for sh in wl.low_pressure_steps()) * geo.n_layers
+
+
+def cpu_baseline(W, cache, torch, args):
+    from oracle import attention as oa
+    geo = W.geo
+    kc = cache["k"].float().cpu().numpy()
+    vc = cache["v"].float().cpu().numpy()
+    table = np.array([W.perm[: wl.blocks_for(W.prompt)]], dtype=np.int64)
+    workers = oa.default_workers()
+    budget_s = args.cpu_seconds
+    total_t, total_pairs, n = 0.0, 0, 0
+    rows = 256
+    while total_t < budget_s and n < 64:
+        dt, pairs = _oracle_sample(kc, vc, table, geo, rows, workers)
+        total_t += dt
+        total_pairs += pairs
+        n += 1
+    us_per_step = total_t / total_pairs * _workload_pairs(geo) * 1e6
+    return {"value": round(us_per_step, 1), "unit": "us", "cores": workers, "kind": "oracle",
+            "sample": f"{n} runs of the oracle on the last {rows} query tokens (all 16 heads) of the "
+                      f"16384-token chunk over its full 16384-token context, {total_t:.1f} s, "
+                      f"extrapolated by causal pair count to the whole step (2 iterations x 36 layers)"}
+
+
+def run_reference(args, rank, world):
+    """The float64 oracle as the reference arm, on this host's cores."""
+    if rank != 0:
+        return None
+    from oracle import attention as oa
+    geo = wl.QWEN25_3B
+    L = 16384
+    nb = wl.blocks_for(L)
+    perm = wl.page_permutation(nb, 0)
+    table = np.array([perm], dtype=np.int64)
+    kc = wl.bf16_normal((nb, geo.n_kv_heads, 16, geo.head_dim), 1, "cpu").float().numpy()
+    vc = wl.bf16_normal((nb, geo.n_kv_heads, 16, geo.head_dim), 2, "cpu").float().numpy()
+    workers = oa.default_workers()
+    rows = 128
+    for _ in range(args.warmup):
+        _oracle_sample(kc, vc, table, geo, rows, workers)
+    total_t, total_pairs = 0.0, 0
+    for _ in range(args.steps):
+        dt, pairs = _oracle_sample(kc, vc, table, geo, rows, workers)
+        total_t += dt
+        total_pairs += pairs
+    us = total_t / total_pairs * _workload_pairs(geo) * 1e6
+    sample = (f"each step: the oracle on the last {rows} query tokens (16 heads) of the 16384-token chunk over its "
+              f"full context; extrapolated by causal pair count to the whole step (2 iterations x 36 layers)")
+    return {"metric": METRIC, "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(us / 1e3, 3), "higher_is_better": False, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": "MBT 16384 low pressure: 25,000-token prompt as chunks (16384, p=0) and "
+                                   "(8616, p=16384); Qwen2.5-3B attention geometry, 36 layers",
+                       "parallelism": "cpu oracle"},
+            "cpu_baseline": {"value": round(us, 1), "unit": "us", "cores": workers, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(us, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    dist = None
+    if world > 1 and args.impl == "ours":
+        import torch
+        import torch.distributed as dist_mod
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", 0)))
+        dist_mod.init_process_group("nccl")
+        dist = dist_mod
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        line = run_ours(args, rank, world, dist)
+    if rank == 0 and line is not None:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -111,6 +111,17 @@ class Scheduler:
         if threshold < 1 or mbt_lo < 1 or mbt_hi < mbt_lo:
             raise ValueError("need threshold >= 1 and 1 <= mbt_lo <= mbt_hi")
         order = sorted(range(len(reqs)), key=lambda i: (reqs[i].arrival_us, i))
+        # a failed plan leaves the pool and every request as they were
+        saved = (deque(self.free), [(r.state, list(r.blocks)) for r in reqs])
+        try:
+            return self._plan(reqs, order, now_us, threshold, mbt_hi, mbt_lo, width)
+        except (OutOfBlocks, ValueError):
+            self.free = saved[0]
+            for r, (st, bl) in zip(reqs, saved[1]):
+                r.state, r.blocks = st, bl
+            raise
+
+    def _plan(self, reqs, order, now_us, threshold, mbt_hi, mbt_lo, width):
 
         # blocks of requests finished in the previous iteration go back to the tail
         for i in order:

@@ -1,0 +1,321 @@
+// Host side of the C ABI: argument checks, TMA descriptors, the split of one
+// attention step into prefill tiles and decode splits, and the launches.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include <cudaTypedefs.h>
+
+#include "ppas_internal.h"
+
+namespace ppas {
+
+namespace {
+
+// Decode rows are split so that one step launches about this many CTAs
+// (two per SM on a 152-SM GB300).  A fixed number keeps the workspace size a
+// pure function of the step's lengths.
+constexpr int64_t kDecodeTargetCtas = 304;
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    });
+    return fn;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+}  // namespace
+
+int32_t device_sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+    static int cached[64] = {0};
+    if (dev >= 0 && dev < 64 && cached[dev]) return cached[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    if (dev >= 0 && dev < 64) cached[dev] = n;
+    return n;
+}
+
+// K or V cache [num_blocks, n_kv_heads, 16, 128] bf16 viewed as rows of 128
+// elements; one TMA box = 16 rows (one page) x 64 columns.
+bool encode_kv_map(CUtensorMap *map, const void *cache, int32_t num_blocks, int32_t n_kv_heads) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(kHeadDim),
+                          static_cast<cuuint64_t>(num_blocks) * n_kv_heads * kPage};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(kRowBytes)};
+    cuuint32_t box[2] = {64, static_cast<cuuint32_t>(kPage)};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(cache), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Q [total_q, n_q_heads, 128] bf16: dims (column, head, token); one box =
+// 128 tokens of one head x 64 columns.
+bool encode_q_map(CUtensorMap *map, const void *q, int32_t total_q, int32_t n_q_heads) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(kHeadDim), static_cast<cuuint64_t>(n_q_heads),
+                          static_cast<cuuint64_t>(total_q)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(kRowBytes),
+                             static_cast<cuuint64_t>(kRowBytes) * n_q_heads};
+    cuuint32_t box[3] = {64, 1, static_cast<cuuint32_t>(kTileQ)};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(q), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                       int32_t n_kv_heads, int32_t /*num_sms*/) {
+    DecodePlan d;
+    int64_t total_pages = 0;
+    for (int32_t s = 0; s < n_seqs; ++s)
+        if (q_lens[s] == 1) {
+            d.rows.push_back(s);
+            total_pages += static_cast<int64_t>((ctx_lens[s] + kPage - 1) / kPage) * n_kv_heads;
+        }
+    if (d.rows.empty()) return d;
+    int64_t pps = (total_pages + kDecodeTargetCtas - 1) / kDecodeTargetCtas;
+    pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
+    pps = (pps + kDecodeWarps - 1) / kDecodeWarps * kDecodeWarps;
+    d.pages_per_split = static_cast<int32_t>(pps);
+    for (int32_t s : d.rows) {
+        const int64_t pages = (ctx_lens[s] + kPage - 1) / kPage;
+        const int32_t ns = static_cast<int32_t>((pages + pps - 1) / pps);
+        d.n_splits.push_back(ns);
+        d.n_part += ns;
+        d.n_ctas += static_cast<int64_t>(ns) * n_kv_heads;
+    }
+    d.ml_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * 2 * sizeof(float));
+    d.o_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * kHeadDim * sizeof(float));
+    d.counter_bytes = align256(d.rows.size() * n_kv_heads * sizeof(int32_t));
+    return d;
+}
+
+}  // namespace ppas
+
+using namespace ppas;
+
+namespace {
+
+ppas_status check_step(const void *q, const void *k_cache, const void *v_cache, int32_t num_blocks,
+                       const int32_t *d_block_tables, int32_t max_blocks_per_seq, const int32_t *h_q_lens,
+                       const int32_t *h_ctx_lens, int32_t n_seqs, int32_t n_q_heads, int32_t n_kv_heads,
+                       int32_t head_dim, const void *out, int64_t *total_q) {
+    if (n_seqs < 0) return PPAS_ERR_INVALID_ARG;
+    if (n_seqs > 0 && (!h_q_lens || !h_ctx_lens)) return PPAS_ERR_INVALID_ARG;
+    if (n_q_heads < 1 || n_kv_heads < 1 || head_dim < 1) return PPAS_ERR_INVALID_ARG;
+    if (head_dim != kHeadDim) return PPAS_ERR_UNSUPPORTED;
+    if (n_q_heads % n_kv_heads != 0) return PPAS_ERR_INVALID_ARG;
+    const int32_t g = n_q_heads / n_kv_heads;
+    if (g != 1 && g != 2 && g != 4 && g != 8) return PPAS_ERR_UNSUPPORTED;
+    int64_t tq = 0;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+        if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return PPAS_ERR_INVALID_ARG;
+        if (static_cast<int64_t>(h_ctx_lens[s]) > static_cast<int64_t>(max_blocks_per_seq) * kPage)
+            return PPAS_ERR_INVALID_ARG;
+        tq += h_q_lens[s];
+    }
+    *total_q = tq;
+    if (n_seqs == 0) return PPAS_OK;
+    if (!q || !k_cache || !v_cache || !d_block_tables || !out) return PPAS_ERR_INVALID_ARG;
+    if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out))
+        return PPAS_ERR_INVALID_ARG;
+    if (num_blocks < 1 || max_blocks_per_seq < 1) return PPAS_ERR_INVALID_ARG;
+    if (tq * n_q_heads > INT32_MAX || static_cast<int64_t>(num_blocks) * n_kv_heads * kPage > INT32_MAX)
+        return PPAS_ERR_UNSUPPORTED;
+    return PPAS_OK;
+}
+
+}  // namespace
+
+extern "C" const char *ppas_status_string(ppas_status s) {
+    switch (s) {
+        case PPAS_OK: return "ok";
+        case PPAS_ERR_INVALID_ARG: return "invalid argument";
+        case PPAS_ERR_CAPACITY: return "capacity exceeded";
+        case PPAS_ERR_OUT_OF_BLOCKS: return "out of KV blocks";
+        case PPAS_ERR_UNSUPPORTED: return "unsupported shape";
+        case PPAS_ERR_CUDA: return "CUDA error";
+        default: return "unknown status";
+    }
+}
+
+extern "C" int32_t ppas_abi_version(void) { return 1; }
+
+extern "C" ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *d_slot_mapping,
+                                      int32_t n_tokens, void *k_cache, void *v_cache, int32_t num_blocks,
+                                      int32_t n_kv_heads, int32_t head_dim, int32_t *d_err_flag, void *stream) {
+    if (n_tokens < 0 || n_kv_heads < 1 || head_dim < 8 || head_dim % 8 != 0 || num_blocks < 1)
+        return PPAS_ERR_INVALID_ARG;
+    if (n_tokens == 0) return PPAS_OK;
+    if (!k_new || !v_new || !d_slot_mapping || !k_cache || !v_cache) return PPAS_ERR_INVALID_ARG;
+    if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
+        return PPAS_ERR_INVALID_ARG;
+    cudaError_t e = launch_kv_append(k_new, v_new, d_slot_mapping, n_tokens, k_cache, v_cache, num_blocks,
+                                     n_kv_heads, head_dim, d_err_flag, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? PPAS_OK : PPAS_ERR_CUDA;
+}
+
+extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
+                                                int32_t n_q_heads, int32_t n_kv_heads) {
+    if (n_seqs <= 0 || !h_q_lens || !h_ctx_lens || n_q_heads < 1 || n_kv_heads < 1) return 0;
+    for (int32_t s = 0; s < n_seqs; ++s)
+        if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return 0;
+    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes();
+}
+
+extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
+                                           int32_t num_blocks, const int32_t *d_block_tables,
+                                           int32_t max_blocks_per_seq, const int32_t *h_q_lens,
+                                           const int32_t *h_ctx_lens, int32_t n_seqs, int32_t n_q_heads,
+                                           int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
+                                           int32_t out_is_fp32, void *workspace, size_t workspace_bytes,
+                                           int32_t *d_err_flag, void *stream) {
+    int64_t total_q = 0;
+    ppas_status st = check_step(q, k_cache, v_cache, num_blocks, d_block_tables, max_blocks_per_seq, h_q_lens,
+                                h_ctx_lens, n_seqs, n_q_heads, n_kv_heads, head_dim, out, &total_q);
+    if (st != PPAS_OK || n_seqs == 0) return st;
+    if (!(scale > 0.f) || !std::isfinite(scale)) return PPAS_ERR_INVALID_ARG;
+    const cudaStream_t cs = static_cast<cudaStream_t>(stream);
+    const int32_t g = n_q_heads / n_kv_heads;
+    const float scale_log2 = scale * 1.4426950408889634f;
+
+    // packed row offsets
+    std::vector<int32_t> q_start(n_seqs);
+    {
+        int32_t acc = 0;
+        for (int32_t s = 0; s < n_seqs; ++s) {
+            q_start[s] = acc;
+            acc += h_q_lens[s];
+        }
+    }
+
+    DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
+    if (dp.total_bytes() > 0) {
+        if (!workspace || workspace_bytes < dp.total_bytes()) return PPAS_ERR_CAPACITY;
+        if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return PPAS_ERR_INVALID_ARG;
+    }
+
+    CUtensorMap tm_k, tm_v;
+    if (!encode_kv_map(&tm_k, k_cache, num_blocks, n_kv_heads) ||
+        !encode_kv_map(&tm_v, v_cache, num_blocks, n_kv_heads))
+        return PPAS_ERR_CUDA;
+
+    // ---------------- decode rows
+    if (!dp.rows.empty()) {
+        uint8_t *ws = static_cast<uint8_t *>(workspace);
+        float *part_ml = reinterpret_cast<float *>(ws);
+        float *part_o = reinterpret_cast<float *>(ws + dp.ml_bytes);
+        int32_t *counters = reinterpret_cast<int32_t *>(ws + dp.ml_bytes + dp.o_bytes);
+        if (cudaMemsetAsync(counters, 0, dp.counter_bytes, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+        DecodeParams dprm;
+        std::memset(&dprm, 0, sizeof(dprm));
+        dprm.q = static_cast<const __nv_bfloat16 *>(q);
+        dprm.block_tables = d_block_tables;
+        dprm.table_stride = max_blocks_per_seq;
+        dprm.num_blocks = num_blocks;
+        dprm.out = out;
+        dprm.out_fp32 = out_is_fp32 ? 1 : 0;
+        dprm.n_q_heads = n_q_heads;
+        dprm.n_kv_heads = n_kv_heads;
+        dprm.group = g;
+        dprm.scale_log2 = scale_log2;
+        dprm.pages_per_split = dp.pages_per_split;
+        dprm.part_ml = part_ml;
+        dprm.part_o = part_o;
+        dprm.err = d_err_flag;
+        int32_t part_base = 0;
+        for (size_t b0 = 0; b0 < dp.rows.size(); b0 += kMaxDecodeRows) {
+            const size_t b1 = std::min(dp.rows.size(), b0 + kMaxDecodeRows);
+            dprm.n_rows = static_cast<int32_t>(b1 - b0);
+            dprm.counters = counters + b0 * n_kv_heads;
+            int32_t cta = 0;
+            for (size_t i = b0; i < b1; ++i) {
+                const int32_t s = dp.rows[i];
+                DecodeRow &r = dprm.rows[i - b0];
+                r.q_row = q_start[s];
+                r.ctx_len = h_ctx_lens[s];
+                r.table_row = s;
+                r.n_splits = dp.n_splits[i];
+                r.cta_base = cta;
+                r.part_base = part_base;
+                cta += r.n_splits * n_kv_heads;
+                part_base += r.n_splits;
+            }
+            dprm.n_ctas = cta;
+            if (launch_decode(tm_k, tm_v, dprm, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+        }
+    }
+
+    // ---------------- prefill chunks
+    struct Tile {
+        int32_t seq, qt, weight;
+    };
+    std::vector<Tile> tiles;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+        if (h_q_lens[s] == 1) continue;
+        const int32_t prefix = h_ctx_lens[s] - h_q_lens[s];
+        const int32_t n_qt = (h_q_lens[s] + kTileQ - 1) / kTileQ;
+        for (int32_t t = 0; t < n_qt; ++t) {
+            const int32_t last = prefix + std::min(h_q_lens[s], (t + 1) * kTileQ) - 1;
+            tiles.push_back({s, t, last / kTileK + 1});
+        }
+    }
+    if (!tiles.empty()) {
+        // heaviest tiles first: the block scheduler hands them out first
+        std::stable_sort(tiles.begin(), tiles.end(), [](const Tile &a, const Tile &b) { return a.weight > b.weight; });
+        CUtensorMap tm_q;
+        if (!encode_q_map(&tm_q, q, static_cast<int32_t>(total_q), n_q_heads)) return PPAS_ERR_CUDA;
+        PrefillParams pp;
+        std::memset(&pp, 0, sizeof(pp));
+        pp.block_tables = d_block_tables;
+        pp.table_stride = max_blocks_per_seq;
+        pp.num_blocks = num_blocks;
+        pp.out = out;
+        pp.out_fp32 = out_is_fp32 ? 1 : 0;
+        pp.n_q_heads = n_q_heads;
+        pp.n_kv_heads = n_kv_heads;
+        pp.group = g;
+        pp.scale_log2 = scale_log2;
+        pp.err = d_err_flag;
+        std::vector<int32_t> local(n_seqs, -1);
+        int32_t n_local = 0;
+        auto flush = [&]() -> bool {
+            if (pp.n_tiles == 0) return true;
+            const bool ok = launch_prefill(tm_q, tm_k, tm_v, pp, cs) == cudaSuccess;
+            pp.n_tiles = 0;
+            std::fill(local.begin(), local.end(), -1);
+            n_local = 0;
+            return ok;
+        };
+        for (const Tile &t : tiles) {
+            if (pp.n_tiles == kMaxPrefillTiles || (local[t.seq] < 0 && n_local == kMaxPrefillSeqs))
+                if (!flush()) return PPAS_ERR_CUDA;
+            if (local[t.seq] < 0) {
+                local[t.seq] = n_local;
+                pp.seqs[n_local] = {q_start[t.seq], h_q_lens[t.seq], h_ctx_lens[t.seq], t.seq};
+                ++n_local;
+            }
+            pp.tiles[pp.n_tiles++] = (static_cast<uint32_t>(local[t.seq]) << 16) | static_cast<uint32_t>(t.qt);
+        }
+        if (!flush()) return PPAS_ERR_CUDA;
+    }
+    return PPAS_OK;
+}

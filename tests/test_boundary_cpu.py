@@ -1,0 +1,90 @@
+"""The C-ABI library loads and exports every entry point ``include/ppas.h``
+declares; host-side argument checks reject bad input before any device work
+(CPU only: no compute call reaches a kernel)."""
+import os
+import re
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def ppas():
+    lib = os.path.join(ROOT, "paper_2608_15171_gb300", "libppas.so")
+    if not os.path.exists(lib):
+        from paper_2608_15171_gb300 import build
+        build.build()
+    from paper_2608_15171_gb300 import ppas as p
+    return p
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "ppas.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ppas_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported(ppas):
+    names = _declared()
+    assert len(names) == 9
+    for n in names:
+        assert hasattr(ppas._lib, n), n
+    assert sorted(ppas.EXPORTED) == names
+
+
+def test_status_strings_and_version(ppas):
+    assert ppas.ppas_abi_version() == 1
+    for code in (0, -1, -2, -3, -4, -5):
+        assert ppas.ppas_status_string(code) != "unknown status"
+
+
+def test_attention_argument_errors_before_device_work(ppas):
+    E = ppas.PpasError
+    ok = dict(q=16, k_cache=16, v_cache=16, num_blocks=4, d_block_tables=16, max_blocks_per_seq=4,
+              q_lens=[2], ctx_lens=[5], n_q_heads=16, n_kv_heads=2, head_dim=128, scale=0.1, out=16,
+              out_is_fp32=False, stream=0)
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        ppas.ppas_attention_step(**a)
+
+    with pytest.raises(E) as e:
+        call(head_dim=64)
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    with pytest.raises(E) as e:
+        call(n_q_heads=12, n_kv_heads=1)
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    with pytest.raises(E) as e:
+        call(n_q_heads=15)
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    for ql, cl in (([0], [5]), ([6], [5]), ([2], [65])):
+        with pytest.raises(E) as e:
+            call(q_lens=ql, ctx_lens=cl)
+        assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    with pytest.raises(E) as e:
+        call(q=8)  # not 16-byte aligned
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    with pytest.raises(E) as e:
+        call(scale=-1.0)
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    # empty step is a no-op
+    call(q_lens=[], ctx_lens=[])
+
+
+def test_kv_append_argument_errors(ppas):
+    with pytest.raises(ppas.PpasError):
+        ppas.ppas_kv_append(16, 16, 16, -1, 16, 16, 4, 2, 128, None, 0)
+    with pytest.raises(ppas.PpasError):
+        ppas.ppas_kv_append(16, 16, 16, 3, 16, 16, 4, 2, 12, None, 0)
+    ppas.ppas_kv_append(16, 16, 16, 0, 16, 16, 4, 2, 128, None, 0)  # no-op
+
+
+def test_workspace_size_is_a_pure_function_of_lengths(ppas):
+    a = ppas.ppas_attention_workspace_size([1, 1, 512], [25000, 25010, 3000], 16, 2)
+    b = ppas.ppas_attention_workspace_size([1, 1, 512], [25000, 25010, 3000], 16, 2)
+    assert a == b and a > 0 and a % 256 == 0
+    assert ppas.ppas_attention_workspace_size([512], [3000], 16, 2) == 0   # no decode rows
+    assert ppas.ppas_attention_workspace_size([], [], 16, 2) == 0
