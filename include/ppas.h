@@ -5,8 +5,9 @@
  * The library is a plain shared object (libppas.so).  Every entry point takes
  * plain host or device pointers and sizes; nothing here mentions a framework
  * type.  The library keeps no global state apart from a per-device cache of
- * driver entry points; the only stateful object is the opaque planner
- * ppas_sched, which owns the free list of KV blocks.
+ * driver entry points and the fixed scratch array of
+ * ppas_attention_step_noalloc; the only stateful object is the opaque
+ * planner ppas_sched, which owns the free list of KV blocks.
  *
  * Ownership: the caller owns every buffer passed in (inputs, caches,
  * outputs, workspace, error flag, plan arrays).  No call allocates device
@@ -196,6 +197,38 @@ ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *
                                 int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
                                 int32_t out_is_fp32, void *workspace, size_t workspace_bytes,
                                 int32_t *d_err_flag, void *stream);
+
+/* ---------------------------------------------------------------------------
+ * Attention step without a caller-provided workspace.  The paper has no
+ * counterpart to this entry point: it exists for callers that may not
+ * allocate device memory at all (a serving loop that gave all of HBM to its
+ * KV-cache pool at start-up and cannot call cudaMalloc afterwards, or a host
+ * program whose device memory belongs to another allocator).
+ *
+ * Same arguments, layouts and results as ppas_attention_step, minus the
+ * workspace: the split-K decode scratch lives in a fixed array of
+ * PPAS_NOALLOC_SCRATCH_BYTES inside the library's device memory, which every
+ * GPU that loads the library holds until the process exits.  The call makes
+ * no cudaMalloc, cudaFree or other allocating call.
+ *  - A step whose scratch (ppas_attention_workspace_size) exceeds
+ *    PPAS_NOALLOC_SCRATCH_BYTES is rejected with PPAS_ERR_CAPACITY before any
+ *    device work.
+ *  - The first call on a device (with scratch to use) looks up the array's
+ *    device address with that device current; make that first call before
+ *    any stream capture.  PPAS_ERR_CUDA if the lookup fails.
+ *  - All calls share one array, which keeps the last call's contents (the
+ *    parts that must start at zero are cleared on the stream by every call).
+ *    Calls whose work overlaps on the GPU (other streams, other host threads)
+ *    race on it: serialise them.
+ * ------------------------------------------------------------------------- */
+#define PPAS_NOALLOC_SCRATCH_BYTES (4 * 1024 * 1024)
+
+ppas_status ppas_attention_step_noalloc(const void *q, const void *k_cache, const void *v_cache,
+                                        int32_t num_blocks, const int32_t *d_block_tables,
+                                        int32_t max_blocks_per_seq, const int32_t *h_q_lens,
+                                        const int32_t *h_ctx_lens, int32_t n_seqs, int32_t n_q_heads,
+                                        int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
+                                        int32_t out_is_fp32, int32_t *d_err_flag, void *stream);
 
 /* Static description of a status code (never NULL). */
 const char *ppas_status_string(ppas_status status);

@@ -20,7 +20,8 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libppas.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["planner.cpp", "attention_step.cu", "kv_append.cu", "attn_prefill.cu", "attn_decode.cu"]
+SOURCES = ["planner.cpp", "attention_step.cu", "kv_append.cu", "attn_prefill.cu", "attn_decode.cu",
+           "attention_noalloc.cu"]
 
 
 def _nvcc() -> str:

@@ -35,7 +35,8 @@ PPAS_REQ_PENDING, PPAS_REQ_WAITING, PPAS_REQ_RUNNING, PPAS_REQ_FINISHED = 0, 1, 
 
 EXPORTED = ("ppas_sched_create", "ppas_sched_destroy", "ppas_sched_free_blocks", "ppas_plan_step",
             "ppas_kv_append", "ppas_attention_workspace_size", "ppas_attention_step",
-            "ppas_status_string", "ppas_abi_version")
+            "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc")
+PPAS_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
 
 
 class ppas_request(ctypes.Structure):
@@ -79,6 +80,11 @@ _lib.ppas_attention_step.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c
                                      _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_size_t,
                                      _c.c_void_p, _c.c_void_p]
 _lib.ppas_attention_step.restype = _c.c_int32
+_lib.ppas_attention_step_noalloc.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p,
+                                             _c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_int32,
+                                             _c.c_int32, _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p,
+                                             _c.c_void_p]
+_lib.ppas_attention_step_noalloc.restype = _c.c_int32
 _lib.ppas_status_string.argtypes = [_c.c_int32]
 _lib.ppas_status_string.restype = _c.c_char_p
 _lib.ppas_abi_version.argtypes = []
@@ -175,6 +181,21 @@ def ppas_attention_step(q, k_cache, v_cache, num_blocks: int, d_block_tables, ma
                                     float(scale), _ptr(out), 1 if out_is_fp32 else 0, _ptr(workspace),
                                     int(workspace_bytes), _ptr(d_err_flag), _stream(stream)),
            "ppas_attention_step")
+
+
+def ppas_attention_step_noalloc(q, k_cache, v_cache, num_blocks: int, d_block_tables, max_blocks_per_seq: int,
+                                q_lens, ctx_lens, n_q_heads: int, n_kv_heads: int, head_dim: int, scale: float,
+                                out, out_is_fp32: bool, d_err_flag=None, stream=None) -> None:
+    """``ppas_attention_step`` for callers that cannot allocate device memory:
+    the split-K scratch is the library's fixed array of
+    ``PPAS_NOALLOC_SCRATCH_BYTES`` (shared by every call; serialise calls)."""
+    ql, cl = _i32(q_lens), _i32(ctx_lens)
+    _check(_lib.ppas_attention_step_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), int(num_blocks),
+                                            _ptr(d_block_tables), int(max_blocks_per_seq), _p32(ql), _p32(cl),
+                                            int(ql.size), int(n_q_heads), int(n_kv_heads), int(head_dim),
+                                            float(scale), _ptr(out), 1 if out_is_fp32 else 0, _ptr(d_err_flag),
+                                            _stream(stream)),
+           "ppas_attention_step_noalloc")
 
 
 # ---------------------------------------------------------------- planner object
