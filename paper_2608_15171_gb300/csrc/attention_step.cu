@@ -293,6 +293,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         pp.n_q_heads = n_q_heads;
         pp.n_kv_heads = n_kv_heads;
         pp.group = g;
+        pp.heads_per_cta = g >= 2 ? 2 : 1;
         pp.scale_log2 = scale_log2;
         pp.err = d_err_flag;
         std::vector<int32_t> local(n_seqs, -1);

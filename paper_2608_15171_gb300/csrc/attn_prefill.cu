@@ -1,14 +1,20 @@
 // Prefill-chunk attention on the 5th-generation tensor cores (tcgen05).
 //
-// One CTA computes O for one 128-token query tile of one q-head:
-//   S = Q K^T            tcgen05.mma, Q and K tiles in shared memory (TMA),
-//                        S accumulated in TMEM (128 lanes x 128 fp32 columns)
-//   online softmax       each thread owns one query row (its TMEM lane),
-//                        fp32, exp2 domain, causal mask by absolute position
-//   O += P V             P written to shared memory as bf16, V via TMA,
-//                        O accumulated in TMEM
-// K/V tiles are 128 keys = eight 16-token pages, fetched page by page through
-// the block table with 2D TMA boxes of 16 rows x 64 columns (128-byte swizzle).
+// One CTA computes O for one 128-token query tile of two q-heads of the same
+// kv-head (one head when the group size is 1); both Q tiles share every K/V
+// tile it loads.  Warp roles (384 threads):
+//   warp 0      TMA producer: Q tiles once, then 64-key K and V tiles (four
+//               16-token pages each, fetched through the block table) into
+//               a 4-stage ring
+//   warp 1      MMA issuer (one thread): S_t = Q_t K^T into TMEM (double
+//               buffered per tile), then O_t += P_t V into TMEM
+//   warps 4-7   softmax for tile 0, warps 8-11 softmax for tile 1: each
+//               thread owns one query row (its TMEM lane), loads its S row,
+//               masks by absolute position, runs the online softmax in fp32
+//               (exp2 domain), writes P (bf16) to shared memory
+// The running max is only raised (and O rescaled in TMEM) when it grows by
+// more than 2^8; until then the stale max keeps every exponent <= 2^8, and
+// the final O / l is exact either way.
 #include <math.h>
 
 #include "ppas_device.cuh"
@@ -17,26 +23,46 @@
 namespace ppas {
 namespace {
 
-constexpr uint32_t kHalf = 16384;                       // 128 rows x 128 B (64 bf16 columns)
-constexpr uint32_t kTileBytes = 2 * kHalf;              // 128 rows x 256 B
-constexpr uint32_t kBoxBytes = kPage * 128;             // 16 rows x 128 B = one TMA box
-constexpr int kStages = 2;
+constexpr int kKT = 64;                    // keys per KV tile
+constexpr int kNS = 4;                     // KV ring depth
+constexpr int kPagesPerTile = kKT / kPage; // 4
+constexpr uint32_t kBox = 2048;            // one TMA box: 16 rows x 128 B
+constexpr uint32_t kQHalf = 16384;         // 128 rows x 128 B (64 columns)
+constexpr uint32_t kQBytes = 2 * kQHalf;
+constexpr uint32_t kKVHalf = 8192;         // 64 rows x 128 B
+constexpr uint32_t kKVBytes = 2 * kKVHalf;
+constexpr uint32_t kPBytes = 16384;        // 128 rows x 64 keys bf16
+
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + kTileBytes;
-constexpr uint32_t kOffV = kOffK + kStages * kTileBytes;
-constexpr uint32_t kOffP = kOffV + kStages * kTileBytes;
-constexpr uint32_t kOffBar = kOffP + kTileBytes;
-// barriers: q, kv[2], s, o (8 B each), then TMEM base address and abort word
-constexpr uint32_t kBarQ = 0, kBarKV = 8, kBarS = 24, kBarO = 32, kTmemSlot = 64;
-constexpr uint32_t kSmemBytes = kOffBar + 128 + 1024;   // + alignment slack
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS = 0, kColO = 128;
+constexpr uint32_t kOffK = kOffQ + 2 * kQBytes;
+constexpr uint32_t kOffV = kOffK + kNS * kKVBytes;
+constexpr uint32_t kOffP = kOffV + kNS * kKVBytes;
+constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
+enum : int {
+    B_Q = 0,
+    B_KFULL = 1,
+    B_KEMPTY = B_KFULL + kNS,
+    B_VFULL = B_KEMPTY + kNS,
+    B_VEMPTY = B_VFULL + kNS,
+    B_SFULL = B_VEMPTY + kNS,  // [tile][buffer]
+    B_SFREE = B_SFULL + 4,     // [tile][buffer]
+    B_PFULL = B_SFREE + 4,     // [tile]
+    B_ODONE = B_PFULL + 2,     // [tile]
+    B_DRAIN = B_ODONE + 2,
+    B_COUNT = B_DRAIN + 1
+};
+constexpr uint32_t kOffTmem = kOffBar + B_COUNT * 8;
+constexpr uint32_t kOffAbort = kOffTmem + 4;
+static_assert(kOffAbort + 4 <= kOffBar + 256, "barrier area");
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;  // + alignment slack
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+constexpr uint32_t kTmemCols = 512;  // S[2 tiles][2 buffers] x 64 cols, O[2 tiles] x 128 cols
+constexpr uint32_t kColO = 256;
+constexpr float kRescaleThreshold = 8.0f;  // log2 units
 
-constexpr uint32_t kIdescQK = idesc_bf16_f32(128, 128, false, false);  // B = K rows, K-major
-constexpr uint32_t kIdescPV = idesc_bf16_f32(128, 128, false, true);   // B = V rows, MN-major
+constexpr uint32_t kIdescQK = idesc_bf16_f32(128, kKT, false, false);  // B = K rows (K-major)
+constexpr uint32_t kIdescPV = idesc_bf16_f32(128, 128, false, true);   // B = V rows (MN-major)
 
-// 32 TMEM columns of this warp's lanes, waiting for completion before the
-// registers are used.
 __device__ __forceinline__ void tmem_ld32_sync(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
     asm volatile(
@@ -64,40 +90,53 @@ __device__ __forceinline__ void tmem_st32_f(uint32_t taddr, const float (&v)[32]
 
 }  // namespace
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(384, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ PrefillParams p) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_s = smem_u32(smem_raw);
     const uint32_t sb = (raw_s + 1023u) & ~1023u;  // 1024-aligned for the 128-byte swizzle
-    uint8_t *const sg = smem_raw + (sb - raw_s);   // generic pointer to the same place
+    uint8_t *const sg = smem_raw + (sb - raw_s);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int h = blockIdx.x % p.n_q_heads;
-    const uint32_t tile = p.tiles[blockIdx.x / p.n_q_heads];
+    const int hpc = p.heads_per_cta;
+    const int slots = p.n_q_heads / hpc;
+    const int h0 = (blockIdx.x % slots) * hpc;
+    const uint32_t tile = p.tiles[blockIdx.x / slots];
     const PrefillSeq sq = p.seqs[tile >> 16];
     const int t0 = static_cast<int>(tile & 0xFFFFu) * kTileQ;
     const int rows_valid = min(kTileQ, sq.q_len - t0);
     const int prefix = sq.ctx_len - sq.q_len;
-    const int kvh = h / p.group;
+    const int kvh = h0 / p.group;
     const int last_pos = prefix + t0 + rows_valid - 1;
-    const int n_kt = last_pos / kTileK + 1;
+    const int n_kt = last_pos / kKT + 1;
     const int32_t *table = p.block_tables + static_cast<int64_t>(sq.table_row) * p.table_stride;
 
-    const uint32_t bar_q = sb + kOffBar + kBarQ, bar_s = sb + kOffBar + kBarS, bar_o = sb + kOffBar + kBarO;
-    auto bar_kv = [&](int st) { return sb + kOffBar + kBarKV + 8u * st; };
-    volatile uint32_t *tmem_slot = reinterpret_cast<volatile uint32_t *>(sg + kOffBar + kTmemSlot);
+    auto bar = [&](int i) { return sb + kOffBar + 8u * static_cast<uint32_t>(i); };
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sg + kOffAbort);
 
-    if (warp == 0) {
-        tmem_alloc(sb + kOffBar + kTmemSlot, kTmemCols);
+    if (warp == 1) {
+        tmem_alloc(sb + kOffTmem, kTmemCols);
         tmem_relinquish();
     }
-    if (tid == 32) {
-        mbar_init(bar_q, 1);
-        mbar_init(bar_kv(0), 1);
-        mbar_init(bar_kv(1), 1);
-        mbar_init(bar_s, 1);
-        mbar_init(bar_o, 1);
+    if (tid == 0) {
+        mbar_init(bar(B_Q), 1);
+        for (int s = 0; s < kNS; ++s) {
+            mbar_init(bar(B_KFULL + s), 1);
+            mbar_init(bar(B_KEMPTY + s), 1);
+            mbar_init(bar(B_VFULL + s), 1);
+            mbar_init(bar(B_VEMPTY + s), 1);
+        }
+        for (int i = 0; i < 4; ++i) {
+            mbar_init(bar(B_SFULL + i), 1);
+            mbar_init(bar(B_SFREE + i), 4);
+        }
+        for (int t = 0; t < 2; ++t) {
+            mbar_init(bar(B_PFULL + t), 4);
+            mbar_init(bar(B_ODONE + t), 1);
+        }
+        mbar_init(bar(B_DRAIN), 1);
+        *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tm_q);
         prefetch_tmap(&tm_k);
@@ -106,188 +145,254 @@ __global__ void __launch_bounds__(128, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sg + kOffTmem);
 
-    // ---- producer (thread 0): one KV tile = up to 8 pages of K and V
-    auto issue_kv = [&](int j) {
-        const int st = j & 1;
-        const uint32_t bar = bar_kv(st);
-        const int first_key = j * kTileK;
-        const int n_pages = min(8, (sq.ctx_len - first_key + kPage - 1) / kPage);
-        mbar_expect_tx(bar, static_cast<uint32_t>(n_pages) * 4u * kBoxBytes);
-        const uint32_t dk = sb + kOffK + st * kTileBytes, dv = sb + kOffV + st * kTileBytes;
-        for (int pg = 0; pg < n_pages; ++pg) {
-            int blk = __ldg(table + j * 8 + pg);
-            if (blk < 0 || blk >= p.num_blocks) {
-                report_error(p.err, PPAS_DEVERR_BAD_INDEX);
-                blk = 0;  // keep the byte count of the barrier consistent
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            mbar_expect_tx(bar(B_Q), static_cast<uint32_t>(hpc) * kQBytes);
+            const int qrow = sq.q_start + t0;
+            for (int t = 0; t < hpc; ++t) {
+                tma_load_3d(sb + kOffQ + t * kQBytes, &tm_q, 0, h0 + t, qrow, bar(B_Q));
+                tma_load_3d(sb + kOffQ + t * kQBytes + kQHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
             }
-            const int row = (blk * p.n_kv_heads + kvh) * kPage;
-            tma_load_2d(dk + pg * kBoxBytes, &tm_k, 0, row, bar);
-            tma_load_2d(dk + kHalf + pg * kBoxBytes, &tm_k, 64, row, bar);
-            tma_load_2d(dv + pg * kBoxBytes, &tm_v, 0, row, bar);
-            tma_load_2d(dv + kHalf + pg * kBoxBytes, &tm_v, 64, row, bar);
-        }
-    };
-
-    if (tid == 0) {
-        mbar_expect_tx(bar_q, kTileBytes);
-        const int qrow = sq.q_start + t0;
-        tma_load_3d(sb + kOffQ, &tm_q, 0, h, qrow, bar_q);
-        tma_load_3d(sb + kOffQ + kHalf, &tm_q, 64, h, qrow, bar_q);
-        issue_kv(0);
-        if (n_kt > 1) issue_kv(1);
-    }
-
-    const int r = warp * 32 + lane;                       // query row of the tile == TMEM lane
-    const int pos = min(prefix + t0 + r, sq.ctx_len - 1); // last key this row may see
-    const uint32_t t_lane = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    float m_run = -INFINITY, l_run = 0.f;
-    bool ok = true;
-    int j = 0;
-
-    for (; j < n_kt; ++j) {
-        const int st = j & 1;
-        bool w_ok = mbar_wait(bar_kv(st), (j >> 1) & 1, p.err);
-        if (j == 0) w_ok = w_ok && mbar_wait(bar_q, 0, p.err);
-        // rows of the last page past the context may hold anything; zero the
-        // V rows there so that P = 0 times V stays 0
-        const int first_key = j * kTileK;
-        const int keys_here = min(kTileK, sq.ctx_len - first_key);
-        if (w_ok && (keys_here & (kPage - 1))) {
-            const int pg = keys_here / kPage;
-            const int from = keys_here & (kPage - 1);
-            const int n_chunks = (kPage - from) * 8;  // 16-byte chunks per half
-            uint8_t *vbase = sg + kOffV + st * kTileBytes + pg * kBoxBytes + from * 128;
-            for (int c = tid; c < 2 * n_chunks; c += blockDim.x) {
-                const int half = c / n_chunks, cc = c % n_chunks;
-                *reinterpret_cast<uint4 *>(vbase + half * kHalf + cc * 16) = make_uint4(0, 0, 0, 0);
-            }
-            fence_proxy_async_smem();
-        }
-        tc_fence_before();
-        if (__syncthreads_or(!w_ok)) { ok = false; break; }
-
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t q0 = sb + kOffQ, k0 = sb + kOffK + st * kTileBytes;
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-                const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-                umma_bf16(tmem + kColS, smem_desc_sw128(q0 + off, 16, 1024), smem_desc_sw128(k0 + off, 16, 1024),
-                          kIdescQK, kk > 0);
-            }
-            umma_commit(bar_s);
-        }
-        w_ok = __all_sync(0xffffffffu, mbar_wait(bar_s, j & 1, p.err));
-        tc_fence_after();
-
-        if (w_ok) {
-            // ---- softmax of this row over the 128 keys of tile j
-            float s[128];
-#pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                float v[32];
-                tmem_ld32_sync(t_lane + kColS + c4 * 32, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s[c4 * 32 + i] = v[i];
-            }
-            float mx = -INFINITY;
-#pragma unroll
-            for (int i = 0; i < 128; ++i) {
-                s[i] = (first_key + i <= pos) ? s[i] * p.scale_log2 : -INFINITY;
-                mx = fmaxf(mx, s[i]);
-            }
-            const float m_new = fmaxf(m_run, mx);
-            const float alpha = ex2(m_run - m_new);
-            m_run = m_new;
-            float rs = 0.f;
-#pragma unroll
-            for (int i = 0; i < 128; ++i) {
-                s[i] = ex2(s[i] - m_new);
-                rs += s[i];
-            }
-            l_run = l_run * alpha + rs;
-            if (j > 0) {
-#pragma unroll
-                for (int c4 = 0; c4 < 4; ++c4) {
-                    float v[32];
-                    tmem_ld32_sync(t_lane + kColO + c4 * 32, v);
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] *= alpha;
-                    tmem_st32_f(t_lane + kColO + c4 * 32, v);
+            for (int j = 0; j < n_kt; ++j) {
+                if (*abort_flag) break;
+                const int s = j % kNS;
+                const uint32_t ph = (j / kNS) & 1;
+                const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
+                int rows[kPagesPerTile];
+                for (int pg = 0; pg < n_pages; ++pg) {
+                    int blk = __ldg(table + j * kPagesPerTile + pg);
+                    if (blk < 0 || blk >= p.num_blocks) {
+                        report_error(p.err, PPAS_DEVERR_BAD_INDEX);
+                        blk = 0;  // keep the barrier's byte count consistent
+                    }
+                    rows[pg] = (blk * p.n_kv_heads + kvh) * kPage;
                 }
-                tmem_wait_st();
+                if (j >= kNS && !mbar_wait(bar(B_KEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
+                mbar_expect_tx(bar(B_KFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
+                const uint32_t dk = sb + kOffK + s * kKVBytes;
+                for (int pg = 0; pg < n_pages; ++pg) {
+                    tma_load_2d(dk + pg * kBox, &tm_k, 0, rows[pg], bar(B_KFULL + s));
+                    tma_load_2d(dk + kKVHalf + pg * kBox, &tm_k, 64, rows[pg], bar(B_KFULL + s));
+                }
+                if (j >= kNS && !mbar_wait(bar(B_VEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
+                mbar_expect_tx(bar(B_VFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
+                const uint32_t dv = sb + kOffV + s * kKVBytes;
+                for (int pg = 0; pg < n_pages; ++pg) {
+                    tma_load_2d(dv + pg * kBox, &tm_v, 0, rows[pg], bar(B_VFULL + s));
+                    tma_load_2d(dv + kKVHalf + pg * kBox, &tm_v, 64, rows[pg], bar(B_VFULL + s));
+                }
             }
-            // P (bf16) into the K-major, 128-byte-swizzled A-operand layout
-            uint8_t *prow = sg + kOffP + (r >> 3) * 1024 + (r & 7) * 128;
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            bool ok = mbar_wait(bar(B_Q), 0, p.err);
+            tc_fence_after();
+            auto issue_pv = [&](int i) -> bool {
+                const int s = i % kNS;
+                if (!mbar_wait(bar(B_VFULL + s), (i / kNS) & 1, p.err)) return false;
+                const int chunks = min(kPagesPerTile, (sq.ctx_len - i * kKT + kPage - 1) / kPage);
+                const uint32_t v0 = sb + kOffV + s * kKVBytes;
+                for (int t = 0; t < hpc; ++t) {
+                    if (!mbar_wait(bar(B_PFULL + t), i & 1, p.err)) return false;
+                    tc_fence_after();
+                    const uint32_t p0 = sb + kOffP + t * kPBytes;
+                    for (int kk = 0; kk < chunks; ++kk)
+                        umma_bf16(tmem + kColO + t * 128, smem_desc_sw128(p0 + kk * 32, 16, 1024),
+                                  smem_desc_sw128(v0 + kk * 2048, kKVHalf, 1024), kIdescPV,
+                                  (i > 0 || kk > 0) ? 1u : 0u);
+                    umma_commit(bar(B_ODONE + t));
+                }
+                umma_commit(bar(B_VEMPTY + s));
+                return true;
+            };
+            for (int j = 0; ok && j < n_kt; ++j) {
+                if (*abort_flag) { ok = false; break; }
+                const int s = j % kNS, b = j & 1;
+                if (!mbar_wait(bar(B_KFULL + s), (j / kNS) & 1, p.err)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t k0 = sb + kOffK + s * kKVBytes;
+                for (int t = 0; t < hpc && ok; ++t) {
+                    if (j >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((j >> 1) - 1) & 1, p.err)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t q0 = sb + kOffQ + t * kQBytes;
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const uint32_t qo = (kk >> 2) * kQHalf + (kk & 3) * 32;
+                        const uint32_t ko = (kk >> 2) * kKVHalf + (kk & 3) * 32;
+                        umma_bf16(tmem + t * 128 + b * kKT, smem_desc_sw128(q0 + qo, 16, 1024),
+                                  smem_desc_sw128(k0 + ko, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
+                    }
+                    umma_commit(bar(B_SFULL + 2 * t + b));
+                }
+                if (!ok) break;
+                umma_commit(bar(B_KEMPTY + s));
+                if (j >= 1 && !issue_pv(j - 1)) ok = false;
+            }
+            if (ok) ok = issue_pv(n_kt - 1);
+            if (!ok) *abort_flag = 1;
+            // every MMA issued so far completes before TMEM is released
+            umma_commit(bar(B_DRAIN));
+            mbar_wait(bar(B_DRAIN), 0, p.err);
+        }
+    } else if (warp >= 4 && (warp >> 2) - 1 < hpc) {
+        // ------------------------------------------------------------ softmax warpgroups
+        const int t = (warp >> 2) - 1;
+        const int wq = warp & 3;
+        const int r = wq * 32 + lane;                          // query row == TMEM lane
+        const int pos = min(prefix + t0 + r, sq.ctx_len - 1);  // last key this row may see
+        const int min_pos = prefix + t0;
+        const uint32_t t_lane = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+        const float sl2 = p.scale_log2;
+        float m_used = -INFINITY, l_run = 0.f;
+        bool ok = true;
+        uint8_t *prow = sg + kOffP + t * kPBytes + (r >> 3) * 1024 + (r & 7) * 128;
+
+        for (int j = 0; j < n_kt; ++j) {
+            const int b = j & 1;
+            ok = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(bar(B_SFULL + 2 * t + b), (j >> 1) & 1, p.err));
+            if (!ok) break;
+            tc_fence_after();
+            float s[kKT];
+            {
+                float v[32];
+                tmem_ld32_sync(t_lane + t * 128 + b * kKT, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s[i] = v[i];
+                tmem_ld32_sync(t_lane + t * 128 + b * kKT + 32, v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i) s[32 + i] = v[i];
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(B_SFREE + 2 * t + b));
+
+            const int first_key = j * kKT;
+            if (first_key + kKT - 1 > min_pos) {
+#pragma unroll
+                for (int i = 0; i < kKT; ++i)
+                    if (first_key + i > pos) s[i] = -INFINITY;
+            }
+            float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+#pragma unroll
+            for (int i = 4; i < kKT; i += 4) {
+                mx0 = fmaxf(mx0, s[i]);
+                mx1 = fmaxf(mx1, s[i + 1]);
+                mx2 = fmaxf(mx2, s[i + 2]);
+                mx3 = fmaxf(mx3, s[i + 3]);
+            }
+            const float m_cand = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+            const bool need = m_cand > m_used + kRescaleThreshold;
+            float alpha = 1.f;
+            if (need) {
+                alpha = ex2(m_used - m_cand);
+                m_used = m_cand;
+            }
+            const float neg_m = -m_used;
+            float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
+#pragma unroll
+            for (int i = 0; i < kKT; i += 4) {
+                s[i] = ex2(fmaf(s[i], sl2, neg_m));
+                s[i + 1] = ex2(fmaf(s[i + 1], sl2, neg_m));
+                s[i + 2] = ex2(fmaf(s[i + 2], sl2, neg_m));
+                s[i + 3] = ex2(fmaf(s[i + 3], sl2, neg_m));
+                r0 += s[i];
+                r1 += s[i + 1];
+                r2 += s[i + 2];
+                r3 += s[i + 3];
+            }
+            l_run = l_run * alpha + ((r0 + r1) + (r2 + r3));
+
+            if (j >= 1) {
+                // P_t(j-1) consumed and O_t(j-1) complete
+                ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (j - 1) & 1, p.err));
+                if (!ok) break;
+                tc_fence_after();
+                if (__any_sync(0xffffffffu, need)) {
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        float v[32];
+                        tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] *= alpha;
+                        tmem_st32_f(t_lane + kColO + t * 128 + c4 * 32, v);
+                    }
+                    tmem_wait_st();
+                }
+            }
+            if (t == 0 && j == n_kt - 1) {
+                // rows of the last page past the context may hold anything:
+                // zero them in V so that P = 0 times V stays 0
+                const int keys_here = min(kKT, sq.ctx_len - first_key);
+                if (keys_here & (kPage - 1)) {
+                    const int s_idx = j % kNS;
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar(B_VFULL + s_idx), (j / kNS) & 1, p.err));
+                    if (!ok) break;
+                    const int pg = keys_here / kPage, from = keys_here & (kPage - 1);
+                    const int n = (kPage - from) * 8;  // 16-byte chunks per half
+                    uint8_t *vb = sg + kOffV + s_idx * kKVBytes + pg * kBox + from * 128;
+                    for (int c = r; c < 2 * n; c += 128)
+                        *reinterpret_cast<uint4 *>(vb + (c / n) * kKVHalf + (c % n) * 16) = make_uint4(0, 0, 0, 0);
+                }
+            }
+#pragma unroll
+            for (int c = 0; c < kKT / 8; ++c) {
                 uint4 v;
                 v.x = pack_bf16x2(s[8 * c + 0], s[8 * c + 1]);
                 v.y = pack_bf16x2(s[8 * c + 2], s[8 * c + 3]);
                 v.z = pack_bf16x2(s[8 * c + 4], s[8 * c + 5]);
                 v.w = pack_bf16x2(s[8 * c + 6], s[8 * c + 7]);
-                *reinterpret_cast<uint4 *>(prow + (c >> 3) * kHalf + (((c & 7) ^ (r & 7)) << 4)) = v;
+                *reinterpret_cast<uint4 *>(prow + ((c ^ (r & 7)) << 4)) = v;
             }
             fence_proxy_async_smem();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(B_PFULL + t));
         }
-        tc_fence_before();
-        if (__syncthreads_or(!w_ok)) { ok = false; break; }
 
-        if (tid == 0) {
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (n_kt - 1) & 1, p.err));
+        if (ok) {
             tc_fence_after();
-            const uint32_t p0 = sb + kOffP, v0 = sb + kOffV + st * kTileBytes;
-            const int n_chunks = (keys_here + kPage - 1) / kPage;  // 16-key chunks with a valid key
-            for (int kk = 0; kk < n_chunks; ++kk) {
-                const uint64_t da = smem_desc_sw128(p0 + (kk >> 2) * kHalf + (kk & 3) * 32, 16, 1024);
-                const uint64_t db = smem_desc_sw128(v0 + kk * 2048, kHalf, 1024);
-                umma_bf16(tmem + kColO, da, db, kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            umma_commit(bar_o);
-        }
-        w_ok = mbar_wait(bar_o, j & 1, p.err);
-        tc_fence_after();
-        if (__syncthreads_or(!w_ok)) { ok = false; break; }
-        if (tid == 0 && j + 2 < n_kt) issue_kv(j + 2);
-    }
-
-    if (ok) {
-        // ---- epilogue: O / l for valid rows
-        const float inv_l = 1.f / l_run;
-        const int64_t orow = static_cast<int64_t>(sq.q_start + t0 + r) * p.n_q_heads + h;
+            const float inv_l = 1.f / l_run;
+            const int64_t orow = static_cast<int64_t>(sq.q_start + t0 + r) * p.n_q_heads + h0 + t;
 #pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
-            float v[32];
-            tmem_ld32_sync(t_lane + kColO + c4 * 32, v);
-            if (r < rows_valid) {
-                if (p.out_fp32) {
-                    float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.out) + orow * kHeadDim + c4 * 32);
+            for (int c4 = 0; c4 < 4; ++c4) {
+                float v[32];
+                tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+                if (r < rows_valid) {
+                    if (p.out_fp32) {
+                        float4 *dst =
+                            reinterpret_cast<float4 *>(static_cast<float *>(p.out) + orow * kHeadDim + c4 * 32);
 #pragma unroll
-                    for (int i = 0; i < 8; ++i)
-                        dst[i] = make_float4(v[4 * i] * inv_l, v[4 * i + 1] * inv_l, v[4 * i + 2] * inv_l,
-                                             v[4 * i + 3] * inv_l);
-                } else {
-                    uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) + orow * kHeadDim +
-                                                           c4 * 32);
+                        for (int i = 0; i < 8; ++i)
+                            dst[i] = make_float4(v[4 * i] * inv_l, v[4 * i + 1] * inv_l, v[4 * i + 2] * inv_l,
+                                                 v[4 * i + 3] * inv_l);
+                    } else {
+                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
+                                                               orow * kHeadDim + c4 * 32);
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        dst[i] = make_uint4(pack_bf16x2(v[8 * i] * inv_l, v[8 * i + 1] * inv_l),
-                                            pack_bf16x2(v[8 * i + 2] * inv_l, v[8 * i + 3] * inv_l),
-                                            pack_bf16x2(v[8 * i + 4] * inv_l, v[8 * i + 5] * inv_l),
-                                            pack_bf16x2(v[8 * i + 6] * inv_l, v[8 * i + 7] * inv_l));
+                        for (int i = 0; i < 4; ++i)
+                            dst[i] = make_uint4(pack_bf16x2(v[8 * i] * inv_l, v[8 * i + 1] * inv_l),
+                                                pack_bf16x2(v[8 * i + 2] * inv_l, v[8 * i + 3] * inv_l),
+                                                pack_bf16x2(v[8 * i + 4] * inv_l, v[8 * i + 5] * inv_l),
+                                                pack_bf16x2(v[8 * i + 6] * inv_l, v[8 * i + 7] * inv_l));
+                    }
                 }
             }
+        } else {
+            *abort_flag = 1;
         }
-    } else if (tid == 0) {
-        // drain: copies of tiles j+1, j+2 (issued, never consumed) and the MMAs in flight
-        for (int jj = j; jj < min(j + 2, n_kt); ++jj) mbar_wait(bar_kv(jj & 1), (jj >> 1) & 1, nullptr);
-        mbar_wait(bar_s, j & 1, nullptr);
-        mbar_wait(bar_o, j & 1, nullptr);
     }
+
     tc_fence_before();
     __syncthreads();
-    if (warp == 0) {
+    if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
@@ -303,7 +408,8 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
         attr_set = true;
     }
     if (p.n_tiles <= 0) return cudaSuccess;
-    prefill_attn_kernel<<<p.n_tiles * p.n_q_heads, 128, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
+    const int grid = p.n_tiles * (p.n_q_heads / p.heads_per_cta);
+    prefill_attn_kernel<<<grid, 384, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
     return cudaGetLastError();
 }
 

@@ -19,8 +19,8 @@ constexpr int kRowBytes = kHeadDim * 2;        // one bf16 K or V row
 constexpr int kPageBytes = kPage * kRowBytes;  // one (block, kv-head) page: 4 KB
 
 // ------------------------------------------------------------------ prefill
-// Rows with q_len > 1.  One CTA computes one 128-token query tile of one
-// q-head against the tile's causal key range.
+// Rows with q_len > 1.  One CTA computes one 128-token query tile of
+// heads_per_cta q-heads of one kv-head against the tile's causal key range.
 constexpr int kTileQ = 128;      // query tokens per tile (tcgen05 M)
 constexpr int kTileK = 128;      // keys per KV tile (tcgen05 N of Q.K^T, K of P.V)
 constexpr int kMaxPrefillSeqs = 128;
@@ -42,9 +42,10 @@ struct PrefillParams {
     int32_t n_q_heads;
     int32_t n_kv_heads;
     int32_t group;       // n_q_heads / n_kv_heads
+    int32_t heads_per_cta;  // 2 when the group has >= 2 heads, else 1
     float scale_log2;    // scale * log2(e)
     int32_t *err;
-    int32_t n_tiles;     // tiles in this launch; grid = n_tiles * n_q_heads
+    int32_t n_tiles;     // tiles in this launch; grid = n_tiles * n_q_heads / heads_per_cta
     uint32_t tiles[kMaxPrefillTiles];  // (seq << 16) | q_tile, heaviest first
     PrefillSeq seqs[kMaxPrefillSeqs];
 };
