@@ -2,19 +2,22 @@
 //
 // One CTA computes O for one 128-token query tile of two q-heads of the same
 // kv-head (one head when the group size is 1); both Q tiles share every K/V
-// tile it loads.  Warp roles (384 threads):
-//   warp 0      TMA producer: Q tiles once, then 64-key K and V tiles (four
-//               16-token pages each, fetched through the block table) into
-//               a 4-stage ring
-//   warp 1      MMA issuer (one thread): S_t = Q_t K^T into TMEM (double
-//               buffered per tile), then O_t += P_t V into TMEM
-//   warps 4-7   softmax for tile 0, warps 8-11 softmax for tile 1: each
+// tile it loads.  Warp roles (512 threads, four warpgroups):
+//   warps 0-3   TMA producers: warp w owns ring stage w and fetches the
+//               64-key K and V tiles j = w, w+4, ... (four 16-token pages
+//               each, through the block table); warp 0 also loads Q.  One
+//               issuing thread moves only ~7 B/clk of small TMA boxes on
+//               GB300, so the ring is filled by four threads in parallel.
+//   warps 4, 5  MMA issuers, one thread per Q tile: S_t = Q_t K^T into TMEM
+//               (double buffered, one KV tile ahead), then O_t += P_t V
+//   warps 8-11  softmax for tile 0, warps 12-15 softmax for tile 1: each
 //               thread owns one query row (its TMEM lane), loads its S row,
 //               masks by absolute position, runs the online softmax in fp32
 //               (exp2 domain), writes P (bf16) to shared memory
-// The running max is only raised (and O rescaled in TMEM) when it grows by
-// more than 2^8; until then the stale max keeps every exponent <= 2^8, and
-// the final O / l is exact either way.
+// Registers move from the producer/MMA warpgroups to the softmax warpgroups
+// with setmaxnreg.  The running max is only raised (and O rescaled in TMEM)
+// when it grows by more than 2^8; until then the stale max keeps every
+// exponent <= 2^8, and the final O / l is exact either way.
 #include <math.h>
 
 #include "ppas_device.cuh"
@@ -59,6 +62,14 @@ static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 constexpr uint32_t kTmemCols = 512;  // S[2 tiles][2 buffers] x 64 cols, O[2 tiles] x 128 cols
 constexpr uint32_t kColO = 256;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
+constexpr int kThreads = 512;
+constexpr int kProducerWarps = kNS;        // warps 0..3, one per ring stage
+constexpr int kMmaWarp = 4;                // warps 4..7 form the MMA warpgroup
+constexpr int kSoftmaxWarp0 = 8;           // warps 8..11 tile 0, 12..15 tile 1
+// register split: 8 warps x 56 + 8 warps x 200 = 512 threads x 128 at launch
+constexpr int kRegsSmall = 56;
+constexpr int kRegsLarge = 200;
+static_assert(8 * 32 * kRegsSmall + 8 * 32 * kRegsLarge <= kThreads * 128, "register split");
 
 constexpr uint32_t kIdescQK = idesc_bf16_f32(128, kKT, false, false);  // B = K rows (K-major)
 constexpr uint32_t kIdescPV = idesc_bf16_f32(128, 128, false, true);   // B = V rows (MN-major)
@@ -81,6 +92,32 @@ __device__ __forceinline__ void tmem_ld32_sync(uint32_t taddr, float (&v)[32]) {
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 64 TMEM columns of this warp's lanes (one S row per thread), waiting for
+// completion before the registers are used.
+__device__ __forceinline__ void tmem_ld64_sync(uint32_t taddr, float (&v)[64]) {
+    uint32_t r[64];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,"
+        "%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+        "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+          "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]),
+          "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]),
+          "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]),
+          "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]),
+          "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(taddr)
+        : "memory");
+#pragma unroll
+    for (int i = 0; i < 64; ++i) v[i] = __uint_as_float(r[i]);
+}
+
 __device__ __forceinline__ void tmem_st32_f(uint32_t taddr, const float (&v)[32]) {
     uint32_t r[32];
 #pragma unroll
@@ -90,7 +127,7 @@ __device__ __forceinline__ void tmem_st32_f(uint32_t taddr, const float (&v)[32]
 
 }  // namespace
 
-__global__ void __launch_bounds__(384, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                         const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ PrefillParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -115,7 +152,7 @@ __global__ void __launch_bounds__(384, 1)
     auto bar = [&](int i) { return sb + kOffBar + 8u * static_cast<uint32_t>(i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sg + kOffAbort);
 
-    if (warp == 1) {
+    if (warp == kMmaWarp) {
         tmem_alloc(sb + kOffTmem, kTmemCols);
         tmem_relinquish();
     }
@@ -123,9 +160,9 @@ __global__ void __launch_bounds__(384, 1)
         mbar_init(bar(B_Q), 1);
         for (int s = 0; s < kNS; ++s) {
             mbar_init(bar(B_KFULL + s), 1);
-            mbar_init(bar(B_KEMPTY + s), 1);
+            mbar_init(bar(B_KEMPTY + s), hpc);  // one release per tile's MMA thread
             mbar_init(bar(B_VFULL + s), 1);
-            mbar_init(bar(B_VEMPTY + s), 1);
+            mbar_init(bar(B_VEMPTY + s), hpc);
         }
         for (int i = 0; i < 4; ++i) {
             mbar_init(bar(B_SFULL + i), 1);
@@ -135,7 +172,7 @@ __global__ void __launch_bounds__(384, 1)
             mbar_init(bar(B_PFULL + t), 4);
             mbar_init(bar(B_ODONE + t), 1);
         }
-        mbar_init(bar(B_DRAIN), 1);
+        mbar_init(bar(B_DRAIN), hpc);
         *abort_flag = 0;
         fence_mbar_init();
         prefetch_tmap(&tm_q);
@@ -147,103 +184,130 @@ __global__ void __launch_bounds__(384, 1)
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sg + kOffTmem);
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ TMA producer
+    if (warp < kProducerWarps) {
+        // ------------------------------------------------------------ TMA producers
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsSmall));
         if (lane == 0) {
-            mbar_expect_tx(bar(B_Q), static_cast<uint32_t>(hpc) * kQBytes);
-            const int qrow = sq.q_start + t0;
-            for (int t = 0; t < hpc; ++t) {
-                tma_load_3d(sb + kOffQ + t * kQBytes, &tm_q, 0, h0 + t, qrow, bar(B_Q));
-                tma_load_3d(sb + kOffQ + t * kQBytes + kQHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
+            if (warp == 0) {
+                mbar_expect_tx(bar(B_Q), static_cast<uint32_t>(hpc) * kQBytes);
+                const int qrow = sq.q_start + t0;
+                for (int t = 0; t < hpc; ++t) {
+                    tma_load_3d(sb + kOffQ + t * kQBytes, &tm_q, 0, h0 + t, qrow, bar(B_Q));
+                    tma_load_3d(sb + kOffQ + t * kQBytes + kQHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
+                }
             }
-            for (int j = 0; j < n_kt; ++j) {
-                if (*abort_flag) break;
-                const int s = j % kNS;
+            const int s = warp;  // this warp's ring stage: tiles j = s, s + kNS, ...
+            const uint32_t dk = sb + kOffK + s * kKVBytes, dv = sb + kOffV + s * kKVBytes;
+            // page ids of the next tile are loaded while the current one is issued
+            auto load_ids = [&](int j, int (&ids)[kPagesPerTile]) {
+                const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
+#pragma unroll
+                for (int pg = 0; pg < kPagesPerTile; ++pg)
+                    ids[pg] = (j < n_kt && pg < n_pages) ? __ldg(table + j * kPagesPerTile + pg) : 0;
+            };
+            int ids[kPagesPerTile];
+            load_ids(s, ids);
+            for (int j = s; j < n_kt; j += kNS) {
                 const uint32_t ph = (j / kNS) & 1;
                 const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
                 int rows[kPagesPerTile];
-                for (int pg = 0; pg < n_pages; ++pg) {
-                    int blk = __ldg(table + j * kPagesPerTile + pg);
-                    if (blk < 0 || blk >= p.num_blocks) {
+#pragma unroll
+                for (int pg = 0; pg < kPagesPerTile; ++pg) {
+                    int blk = ids[pg];
+                    if (pg < n_pages && (blk < 0 || blk >= p.num_blocks)) {
                         report_error(p.err, PPAS_DEVERR_BAD_INDEX);
                         blk = 0;  // keep the barrier's byte count consistent
                     }
                     rows[pg] = (blk * p.n_kv_heads + kvh) * kPage;
                 }
+                load_ids(j + kNS, ids);
                 if (j >= kNS && !mbar_wait(bar(B_KEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
                 mbar_expect_tx(bar(B_KFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
-                const uint32_t dk = sb + kOffK + s * kKVBytes;
                 for (int pg = 0; pg < n_pages; ++pg) {
                     tma_load_2d(dk + pg * kBox, &tm_k, 0, rows[pg], bar(B_KFULL + s));
                     tma_load_2d(dk + kKVHalf + pg * kBox, &tm_k, 64, rows[pg], bar(B_KFULL + s));
                 }
                 if (j >= kNS && !mbar_wait(bar(B_VEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
                 mbar_expect_tx(bar(B_VFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
-                const uint32_t dv = sb + kOffV + s * kKVBytes;
                 for (int pg = 0; pg < n_pages; ++pg) {
                     tma_load_2d(dv + pg * kBox, &tm_v, 0, rows[pg], bar(B_VFULL + s));
                     tma_load_2d(dv + kKVHalf + pg * kBox, &tm_v, 64, rows[pg], bar(B_VFULL + s));
                 }
             }
         }
-    } else if (warp == 1) {
-        // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+    } else if (warp < kSoftmaxWarp0) {
+        // ------------------------------------------------------------ MMA issuers
+        // lane 0 of warp kMmaWarp + t issues every MMA of Q tile t; the two
+        // threads share only the K/V stages, which each releases once
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsSmall));
+        const int t = warp - kMmaWarp;
+        if (t < hpc && lane == 0) {
             bool ok = mbar_wait(bar(B_Q), 0, p.err);
             tc_fence_after();
+            // descriptors are built once; advancing one operand by b bytes
+            // adds b >> 4 to the start-address field (no carry: < 256 KB)
+            const uint64_t dq = smem_desc_sw128(sb + kOffQ + t * kQBytes, 16, 1024);
+            const uint64_t dk0 = smem_desc_sw128(sb + kOffK, 16, 1024);
+            const uint64_t dv0 = smem_desc_sw128(sb + kOffV, kKVHalf, 1024);
+            const uint64_t dp = smem_desc_sw128(sb + kOffP + t * kPBytes, 16, 1024);
+            const uint32_t d_s = tmem + t * 128, d_o = tmem + kColO + t * 128;
+            // S_t(j) = Q_t K(j)^T into S buffer j % 2 of this tile
+            auto issue_qk = [&](int j) -> bool {
+                const int s = j % kNS, b = j & 1;
+                if (!mbar_wait(bar(B_KFULL + s), (j / kNS) & 1, p.err)) return false;
+                // the softmax has read S_t(j-2) out of this buffer
+                if (j >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((j >> 1) - 1) & 1, p.err)) return false;
+                tc_fence_after();
+                const uint64_t dk = dk0 + ((s * kKVBytes) >> 4);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint32_t qo = (kk >> 2) * kQHalf + (kk & 3) * 32;
+                    const uint32_t ko = (kk >> 2) * kKVHalf + (kk & 3) * 32;
+                    umma_bf16(d_s + b * kKT, dq + (qo >> 4), dk + (ko >> 4), kIdescQK, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(bar(B_SFULL + 2 * t + b));
+                umma_commit(bar(B_KEMPTY + s));
+                return true;
+            };
+            // O_t += P_t(i) V(i)
             auto issue_pv = [&](int i) -> bool {
                 const int s = i % kNS;
                 if (!mbar_wait(bar(B_VFULL + s), (i / kNS) & 1, p.err)) return false;
+                if (!mbar_wait(bar(B_PFULL + t), i & 1, p.err)) return false;
+                tc_fence_after();
                 const int chunks = min(kPagesPerTile, (sq.ctx_len - i * kKT + kPage - 1) / kPage);
-                const uint32_t v0 = sb + kOffV + s * kKVBytes;
-                for (int t = 0; t < hpc; ++t) {
-                    if (!mbar_wait(bar(B_PFULL + t), i & 1, p.err)) return false;
-                    tc_fence_after();
-                    const uint32_t p0 = sb + kOffP + t * kPBytes;
-                    for (int kk = 0; kk < chunks; ++kk)
-                        umma_bf16(tmem + kColO + t * 128, smem_desc_sw128(p0 + kk * 32, 16, 1024),
-                                  smem_desc_sw128(v0 + kk * 2048, kKVHalf, 1024), kIdescPV,
+                const uint64_t dv = dv0 + ((s * kKVBytes) >> 4);
+                if (chunks == kPagesPerTile) {
+#pragma unroll
+                    for (int kk = 0; kk < kPagesPerTile; ++kk)
+                        umma_bf16(d_o, dp + ((kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescPV,
                                   (i > 0 || kk > 0) ? 1u : 0u);
-                    umma_commit(bar(B_ODONE + t));
+                } else {
+                    for (int kk = 0; kk < chunks; ++kk)
+                        umma_bf16(d_o, dp + ((kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescPV,
+                                  (i > 0 || kk > 0) ? 1u : 0u);
                 }
+                umma_commit(bar(B_ODONE + t));
                 umma_commit(bar(B_VEMPTY + s));
                 return true;
             };
+            // Q K^T runs one KV tile ahead of P V, so the next S is ready when
+            // the softmax warpgroup finishes the current one
+            if (ok) ok = issue_qk(0);
             for (int j = 0; ok && j < n_kt; ++j) {
-                if (*abort_flag) { ok = false; break; }
-                const int s = j % kNS, b = j & 1;
-                if (!mbar_wait(bar(B_KFULL + s), (j / kNS) & 1, p.err)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t k0 = sb + kOffK + s * kKVBytes;
-                for (int t = 0; t < hpc && ok; ++t) {
-                    if (j >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((j >> 1) - 1) & 1, p.err)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t q0 = sb + kOffQ + t * kQBytes;
-#pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        const uint32_t qo = (kk >> 2) * kQHalf + (kk & 3) * 32;
-                        const uint32_t ko = (kk >> 2) * kKVHalf + (kk & 3) * 32;
-                        umma_bf16(tmem + t * 128 + b * kKT, smem_desc_sw128(q0 + qo, 16, 1024),
-                                  smem_desc_sw128(k0 + ko, 16, 1024), kIdescQK, kk > 0 ? 1u : 0u);
-                    }
-                    umma_commit(bar(B_SFULL + 2 * t + b));
-                }
-                if (!ok) break;
-                umma_commit(bar(B_KEMPTY + s));
-                if (j >= 1 && !issue_pv(j - 1)) ok = false;
+                if (j + 1 < n_kt && !issue_qk(j + 1)) { ok = false; break; }
+                if (!issue_pv(j)) ok = false;
             }
-            if (ok) ok = issue_pv(n_kt - 1);
             if (!ok) *abort_flag = 1;
             // every MMA issued so far completes before TMEM is released
             umma_commit(bar(B_DRAIN));
             mbar_wait(bar(B_DRAIN), 0, p.err);
         }
-    } else if (warp >= 4 && (warp >> 2) - 1 < hpc) {
+    } else {
         // ------------------------------------------------------------ softmax warpgroups
-        const int t = (warp >> 2) - 1;
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsLarge));
+      if ((warp - kSoftmaxWarp0) / 4 < hpc) {
+        const int t = (warp - kSoftmaxWarp0) / 4;
         const int wq = warp & 3;
         const int r = wq * 32 + lane;                          // query row == TMEM lane
         const int pos = min(prefix + t0 + r, sq.ctx_len - 1);  // last key this row may see
@@ -260,15 +324,7 @@ __global__ void __launch_bounds__(384, 1)
             if (!ok) break;
             tc_fence_after();
             float s[kKT];
-            {
-                float v[32];
-                tmem_ld32_sync(t_lane + t * 128 + b * kKT, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s[i] = v[i];
-                tmem_ld32_sync(t_lane + t * 128 + b * kKT + 32, v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i) s[32 + i] = v[i];
-            }
+            tmem_ld64_sync(t_lane + t * 128 + b * kKT, s);
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(B_SFREE + 2 * t + b));
@@ -326,9 +382,12 @@ __global__ void __launch_bounds__(384, 1)
                     tmem_wait_st();
                 }
             }
-            if (t == 0 && j == n_kt - 1) {
+            if (j == n_kt - 1) {
                 // rows of the last page past the context may hold anything:
-                // zero them in V so that P = 0 times V stays 0
+                // zero them in V so that P = 0 times V stays 0.  Each tile's
+                // warpgroup does it before releasing its own P, so both P V
+                // products are ordered after it (the second writes the same
+                // zeros again)
                 const int keys_here = min(kKT, sq.ctx_len - first_key);
                 if (keys_here & (kPage - 1)) {
                     const int s_idx = j % kNS;
@@ -388,11 +447,12 @@ __global__ void __launch_bounds__(384, 1)
         } else {
             *abort_flag = 1;
         }
+      }
     }
 
     tc_fence_before();
     __syncthreads();
-    if (warp == 1) {
+    if (warp == kMmaWarp) {
         tc_fence_after();
         tmem_dealloc(tmem, kTmemCols);
     }
@@ -409,7 +469,7 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
     }
     if (p.n_tiles <= 0) return cudaSuccess;
     const int grid = p.n_tiles * (p.n_q_heads / p.heads_per_cta);
-    prefill_attn_kernel<<<grid, 384, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
+    prefill_attn_kernel<<<grid, kThreads, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
     return cudaGetLastError();
 }
 
