@@ -49,16 +49,17 @@ extern "C" ppas_status ppas_attention_step_noalloc(const void *q, const void *k_
                                                    const int32_t *h_ctx_lens, int32_t n_seqs, int32_t n_q_heads,
                                                    int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
                                                    int32_t out_is_fp32, int32_t *d_err_flag, void *stream) {
-    // the scratch this step needs must fit the fixed array (checked before any CUDA call)
-    const size_t need = ppas_attention_workspace_size(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
+    // the scratch this step needs must fit the fixed array (checked before any
+    // CUDA call); prefill tiles run unsplit when their split partials do not fit
+    const size_t need = ppas::workspace_min_size(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
     if (need > static_cast<size_t>(PPAS_NOALLOC_SCRATCH_BYTES)) return PPAS_ERR_CAPACITY;
     void *scratch = nullptr;
-    if (need > 0) {
+    if (n_seqs > 0) {
         scratch = scratch_on_current_device();
         if (!scratch) return PPAS_ERR_CUDA;
     }
     // the step itself is the ordinary one, with the fixed array as its workspace
     return ppas_attention_step(q, k_cache, v_cache, num_blocks, d_block_tables, max_blocks_per_seq, h_q_lens,
                                h_ctx_lens, n_seqs, n_q_heads, n_kv_heads, head_dim, scale, out, out_is_fp32, scratch,
-                               need > 0 ? static_cast<size_t>(PPAS_NOALLOC_SCRATCH_BYTES) : 0, d_err_flag, stream);
+                               scratch ? static_cast<size_t>(PPAS_NOALLOC_SCRATCH_BYTES) : 0, d_err_flag, stream);
 }

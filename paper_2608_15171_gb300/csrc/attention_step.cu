@@ -108,6 +108,60 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
     return d;
 }
 
+PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                         int32_t n_kv_heads, bool allow_split) {
+    PrefillPlan pf;
+    const int32_t g = n_q_heads / n_kv_heads;
+    pf.heads_per_cta = g >= 2 ? 2 : 1;
+    pf.slots = n_q_heads / pf.heads_per_cta;
+    struct Tile {
+        int32_t seq, qt, n_kt;
+    };
+    std::vector<Tile> tiles;
+    int64_t total = 0;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+        if (q_lens[s] == 1) continue;
+        const int32_t prefix = ctx_lens[s] - q_lens[s];
+        const int32_t n_qt = (q_lens[s] + kTileQ - 1) / kTileQ;
+        for (int32_t t = 0; t < n_qt; ++t) {
+            const int32_t last = prefix + std::min(q_lens[s], (t + 1) * kTileQ) - 1;
+            tiles.push_back({s, t, last / kPrefillKT + 1});
+            total += static_cast<int64_t>(last / kPrefillKT + 1) * pf.slots;
+        }
+    }
+    int64_t per_cta = (total + kPrefillTargetCtas - 1) / kPrefillTargetCtas;
+    per_cta = std::max<int64_t>(per_cta, kPrefillMinSplitTiles);
+    for (const Tile &t : tiles) {
+        int32_t ns = 1;
+        if (allow_split)
+            ns = static_cast<int32_t>(std::min<int64_t>(kPrefillMaxSplits, (t.n_kt + per_cta - 1) / per_cta));
+        const int32_t part = ns > 1 ? static_cast<int32_t>(pf.n_part) : -1;
+        for (int32_t i = 0; i < ns; ++i) {
+            const int32_t kt0 = static_cast<int32_t>(static_cast<int64_t>(t.n_kt) * i / ns);
+            const int32_t kt1 = static_cast<int32_t>(static_cast<int64_t>(t.n_kt) * (i + 1) / ns);
+            pf.items.push_back({t.seq, t.qt, kt0, kt1, part, i, ns});
+        }
+        if (ns > 1) pf.n_part += ns;
+    }
+    // heaviest first: the block scheduler hands them out first
+    std::stable_sort(pf.items.begin(), pf.items.end(), [](const PrefillItem &a, const PrefillItem &b) {
+        return (a.kt1 - a.kt0) > (b.kt1 - b.kt0);
+    });
+    const size_t per_part = static_cast<size_t>(pf.slots) * pf.heads_per_cta * kTileQ;
+    pf.o_bytes = align256(static_cast<size_t>(pf.n_part) * per_part * kHeadDim * sizeof(float));
+    pf.ml_bytes = align256(static_cast<size_t>(pf.n_part) * per_part * 2 * sizeof(float));
+    pf.ticket_bytes = align256(static_cast<size_t>(pf.n_part) * pf.slots * sizeof(int32_t));
+    return pf;
+}
+
+size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                          int32_t n_kv_heads) {
+    if (n_seqs <= 0 || !q_lens || !ctx_lens || n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads) return 0;
+    for (int32_t s = 0; s < n_seqs; ++s)
+        if (q_lens[s] < 1 || ctx_lens[s] < q_lens[s]) return 0;
+    return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes();
+}
+
 }  // namespace ppas
 
 using namespace ppas;
@@ -175,10 +229,12 @@ extern "C" ppas_status ppas_kv_append(const void *k_new, const void *v_new, cons
 
 extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
                                                 int32_t n_q_heads, int32_t n_kv_heads) {
-    if (n_seqs <= 0 || !h_q_lens || !h_ctx_lens || n_q_heads < 1 || n_kv_heads < 1) return 0;
+    if (n_seqs <= 0 || !h_q_lens || !h_ctx_lens || n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads)
+        return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return 0;
-    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes();
+    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes() +
+           plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true).total_bytes();
 }
 
 extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
@@ -208,8 +264,13 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     }
 
     DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
-    if (dp.total_bytes() > 0) {
-        if (!workspace || workspace_bytes < dp.total_bytes()) return PPAS_ERR_CAPACITY;
+    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true);
+    // a workspace too small for the prefill splits runs the prefill tiles unsplit
+    if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
+        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false);
+    const size_t need = dp.total_bytes() + pf.total_bytes();
+    if (need > 0) {
+        if (!workspace || workspace_bytes < need) return PPAS_ERR_CAPACITY;
         if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return PPAS_ERR_INVALID_ARG;
     }
 
@@ -265,24 +326,10 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     }
 
     // ---------------- prefill chunks
-    struct Tile {
-        int32_t seq, qt, weight;
-    };
-    std::vector<Tile> tiles;
-    for (int32_t s = 0; s < n_seqs; ++s) {
-        if (h_q_lens[s] == 1) continue;
-        const int32_t prefix = h_ctx_lens[s] - h_q_lens[s];
-        const int32_t n_qt = (h_q_lens[s] + kTileQ - 1) / kTileQ;
-        for (int32_t t = 0; t < n_qt; ++t) {
-            const int32_t last = prefix + std::min(h_q_lens[s], (t + 1) * kTileQ) - 1;
-            tiles.push_back({s, t, last / kTileK + 1});
-        }
-    }
-    if (!tiles.empty()) {
-        // heaviest tiles first: the block scheduler hands them out first
-        std::stable_sort(tiles.begin(), tiles.end(), [](const Tile &a, const Tile &b) { return a.weight > b.weight; });
+    if (!pf.items.empty()) {
         CUtensorMap tm_q;
         if (!encode_q_map(&tm_q, q, static_cast<int32_t>(total_q), n_q_heads)) return PPAS_ERR_CUDA;
+        uint8_t *pws = static_cast<uint8_t *>(workspace) + dp.total_bytes();
         PrefillParams pp;
         std::memset(&pp, 0, sizeof(pp));
         pp.block_tables = d_block_tables;
@@ -293,28 +340,38 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         pp.n_q_heads = n_q_heads;
         pp.n_kv_heads = n_kv_heads;
         pp.group = g;
-        pp.heads_per_cta = g >= 2 ? 2 : 1;
+        pp.heads_per_cta = pf.heads_per_cta;
         pp.scale_log2 = scale_log2;
         pp.err = d_err_flag;
+        if (pf.n_part > 0) {
+            pp.part_o = reinterpret_cast<float *>(pws);
+            pp.part_ml = reinterpret_cast<float *>(pws + pf.o_bytes);
+            pp.tickets = reinterpret_cast<int32_t *>(pws + pf.o_bytes + pf.ml_bytes);
+            if (cudaMemsetAsync(pp.tickets, 0, pf.ticket_bytes, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+        }
         std::vector<int32_t> local(n_seqs, -1);
         int32_t n_local = 0;
         auto flush = [&]() -> bool {
-            if (pp.n_tiles == 0) return true;
+            if (pp.n_work == 0) return true;
             const bool ok = launch_prefill(tm_q, tm_k, tm_v, pp, cs) == cudaSuccess;
-            pp.n_tiles = 0;
+            pp.n_work = 0;
             std::fill(local.begin(), local.end(), -1);
             n_local = 0;
             return ok;
         };
-        for (const Tile &t : tiles) {
-            if (pp.n_tiles == kMaxPrefillTiles || (local[t.seq] < 0 && n_local == kMaxPrefillSeqs))
+        for (const PrefillItem &it : pf.items) {
+            if (pp.n_work == kMaxPrefillWork || (local[it.seq] < 0 && n_local == kMaxPrefillSeqs))
                 if (!flush()) return PPAS_ERR_CUDA;
-            if (local[t.seq] < 0) {
-                local[t.seq] = n_local;
-                pp.seqs[n_local] = {q_start[t.seq], h_q_lens[t.seq], h_ctx_lens[t.seq], t.seq};
+            if (local[it.seq] < 0) {
+                local[it.seq] = n_local;
+                pp.seqs[n_local] = {q_start[it.seq], h_q_lens[it.seq], h_ctx_lens[it.seq], it.seq};
                 ++n_local;
             }
-            pp.tiles[pp.n_tiles++] = (static_cast<uint32_t>(local[t.seq]) << 16) | static_cast<uint32_t>(t.qt);
+            PrefillWork &w = pp.work[pp.n_work++];
+            w.seq_qt = (static_cast<uint32_t>(local[it.seq]) << 16) | static_cast<uint32_t>(it.qt);
+            w.kt_range = (static_cast<uint32_t>(it.kt0) << 16) | static_cast<uint32_t>(it.kt1);
+            w.part = it.part;
+            w.split = (static_cast<uint32_t>(it.n_splits) << 16) | static_cast<uint32_t>(it.split);
         }
         if (!flush()) return PPAS_ERR_CUDA;
     }

@@ -26,7 +26,7 @@
 namespace ppas {
 namespace {
 
-constexpr int kKT = 64;                    // keys per KV tile
+constexpr int kKT = kPrefillKT;            // keys per KV tile
 constexpr int kNS = 4;                     // KV ring depth
 constexpr int kPagesPerTile = kKT / kPage; // 4
 constexpr uint32_t kBox = 2048;            // one TMA box: 16 rows x 128 B
@@ -125,6 +125,43 @@ __device__ __forceinline__ void tmem_st32_f(uint32_t taddr, const float (&v)[32]
     tmem_st32(taddr, r);
 }
 
+__device__ __forceinline__ void named_barrier_sync(int id, int n) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// barrier over n threads that also ORs a predicate across them
+__device__ __forceinline__ int named_barrier_or(int id, int n, int pred) {
+    int out;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.b32 q, %3, 0;\n\t"
+        "bar.red.or.pred p, %1, %2, q;\n\t"
+        "selp.b32 %0, 1, 0, p;\n\t}"
+        : "=r"(out)
+        : "r"(id), "r"(n), "r"(pred)
+        : "memory");
+    return out;
+}
+
+// 32 consecutive output columns of one row, scaled by inv_l
+__device__ __forceinline__ void store_row32(const PrefillParams &p, int64_t orow, int c4, const float (&v)[32],
+                                            float inv_l) {
+    if (p.out_fp32) {
+        float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.out) + orow * kHeadDim + c4 * 32);
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            dst[i] = make_float4(v[4 * i] * inv_l, v[4 * i + 1] * inv_l, v[4 * i + 2] * inv_l, v[4 * i + 3] * inv_l);
+    } else {
+        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) + orow * kHeadDim + c4 * 32);
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            dst[i] = make_uint4(pack_bf16x2(v[8 * i] * inv_l, v[8 * i + 1] * inv_l),
+                                pack_bf16x2(v[8 * i + 2] * inv_l, v[8 * i + 3] * inv_l),
+                                pack_bf16x2(v[8 * i + 4] * inv_l, v[8 * i + 5] * inv_l),
+                                pack_bf16x2(v[8 * i + 6] * inv_l, v[8 * i + 7] * inv_l));
+    }
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -138,15 +175,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int hpc = p.heads_per_cta;
     const int slots = p.n_q_heads / hpc;
-    const int h0 = (blockIdx.x % slots) * hpc;
-    const uint32_t tile = p.tiles[blockIdx.x / slots];
-    const PrefillSeq sq = p.seqs[tile >> 16];
-    const int t0 = static_cast<int>(tile & 0xFFFFu) * kTileQ;
+    const int slot = blockIdx.x % slots;
+    const int h0 = slot * hpc;
+    const PrefillWork wk = p.work[blockIdx.x / slots];
+    const PrefillSeq sq = p.seqs[wk.seq_qt >> 16];
+    const int t0 = static_cast<int>(wk.seq_qt & 0xFFFFu) * kTileQ;
     const int rows_valid = min(kTileQ, sq.q_len - t0);
     const int prefix = sq.ctx_len - sq.q_len;
     const int kvh = h0 / p.group;
     const int last_pos = prefix + t0 + rows_valid - 1;
-    const int n_kt = last_pos / kKT + 1;
+    const int n_kt_all = last_pos / kKT + 1;           // KV tiles of the whole causal range
+    const int kt0 = static_cast<int>(wk.kt_range >> 16);  // this CTA's range [kt0, kt0 + n_kt)
+    const int n_kt = static_cast<int>(wk.kt_range & 0xFFFFu) - kt0;
+    const int n_splits = static_cast<int>(wk.split >> 16);
     const int32_t *table = p.block_tables + static_cast<int64_t>(sq.table_row) * p.table_stride;
 
     auto bar = [&](int i) { return sb + kOffBar + 8u * static_cast<uint32_t>(i); };
@@ -196,19 +237,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tma_load_3d(sb + kOffQ + t * kQBytes + kQHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
                 }
             }
-            const int s = warp;  // this warp's ring stage: tiles j = s, s + kNS, ...
+            const int s = warp;  // this warp's ring stage: local tiles jj = s, s + kNS, ...
             const uint32_t dk = sb + kOffK + s * kKVBytes, dv = sb + kOffV + s * kKVBytes;
             // page ids of the next tile are loaded while the current one is issued
-            auto load_ids = [&](int j, int (&ids)[kPagesPerTile]) {
+            auto load_ids = [&](int jj, int (&ids)[kPagesPerTile]) {
+                const int j = kt0 + jj;
                 const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
 #pragma unroll
                 for (int pg = 0; pg < kPagesPerTile; ++pg)
-                    ids[pg] = (j < n_kt && pg < n_pages) ? __ldg(table + j * kPagesPerTile + pg) : 0;
+                    ids[pg] = (jj < n_kt && pg < n_pages) ? __ldg(table + j * kPagesPerTile + pg) : 0;
             };
             int ids[kPagesPerTile];
             load_ids(s, ids);
-            for (int j = s; j < n_kt; j += kNS) {
-                const uint32_t ph = (j / kNS) & 1;
+            for (int jj = s; jj < n_kt; jj += kNS) {
+                const int j = kt0 + jj;
+                const uint32_t ph = (jj / kNS) & 1;
                 const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
                 int rows[kPagesPerTile];
 #pragma unroll
@@ -220,14 +263,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     rows[pg] = (blk * p.n_kv_heads + kvh) * kPage;
                 }
-                load_ids(j + kNS, ids);
-                if (j >= kNS && !mbar_wait(bar(B_KEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
+                load_ids(jj + kNS, ids);
+                if (jj >= kNS && !mbar_wait(bar(B_KEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
                 mbar_expect_tx(bar(B_KFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
                 for (int pg = 0; pg < n_pages; ++pg) {
                     tma_load_2d(dk + pg * kBox, &tm_k, 0, rows[pg], bar(B_KFULL + s));
                     tma_load_2d(dk + kKVHalf + pg * kBox, &tm_k, 64, rows[pg], bar(B_KFULL + s));
                 }
-                if (j >= kNS && !mbar_wait(bar(B_VEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
+                if (jj >= kNS && !mbar_wait(bar(B_VEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
                 mbar_expect_tx(bar(B_VFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
                 for (int pg = 0; pg < n_pages; ++pg) {
                     tma_load_2d(dv + pg * kBox, &tm_v, 0, rows[pg], bar(B_VFULL + s));
@@ -251,12 +294,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t dv0 = smem_desc_sw128(sb + kOffV, kKVHalf, 1024);
             const uint64_t dp = smem_desc_sw128(sb + kOffP + t * kPBytes, 16, 1024);
             const uint32_t d_s = tmem + t * 128, d_o = tmem + kColO + t * 128;
-            // S_t(j) = Q_t K(j)^T into S buffer j % 2 of this tile
-            auto issue_qk = [&](int j) -> bool {
-                const int s = j % kNS, b = j & 1;
-                if (!mbar_wait(bar(B_KFULL + s), (j / kNS) & 1, p.err)) return false;
-                // the softmax has read S_t(j-2) out of this buffer
-                if (j >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((j >> 1) - 1) & 1, p.err)) return false;
+            // S_t(jj) = Q_t K(kt0 + jj)^T into S buffer jj % 2 of this tile
+            auto issue_qk = [&](int jj) -> bool {
+                const int s = jj % kNS, b = jj & 1;
+                if (!mbar_wait(bar(B_KFULL + s), (jj / kNS) & 1, p.err)) return false;
+                // the softmax has read S_t(jj-2) out of this buffer
+                if (jj >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((jj >> 1) - 1) & 1, p.err)) return false;
                 tc_fence_after();
                 const uint64_t dk = dk0 + ((s * kKVBytes) >> 4);
 #pragma unroll
@@ -269,13 +312,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 umma_commit(bar(B_KEMPTY + s));
                 return true;
             };
-            // O_t += P_t(i) V(i)
+            // O_t += P_t(i) V(kt0 + i)
             auto issue_pv = [&](int i) -> bool {
                 const int s = i % kNS;
                 if (!mbar_wait(bar(B_VFULL + s), (i / kNS) & 1, p.err)) return false;
                 if (!mbar_wait(bar(B_PFULL + t), i & 1, p.err)) return false;
                 tc_fence_after();
-                const int chunks = min(kPagesPerTile, (sq.ctx_len - i * kKT + kPage - 1) / kPage);
+                const int chunks = min(kPagesPerTile, (sq.ctx_len - (kt0 + i) * kKT + kPage - 1) / kPage);
                 const uint64_t dv = dv0 + ((s * kKVBytes) >> 4);
                 if (chunks == kPagesPerTile) {
 #pragma unroll
@@ -318,9 +361,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         uint8_t *prow = sg + kOffP + t * kPBytes + (r >> 3) * 1024 + (r & 7) * 128;
 
-        for (int j = 0; j < n_kt; ++j) {
-            const int b = j & 1;
-            ok = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(bar(B_SFULL + 2 * t + b), (j >> 1) & 1, p.err));
+        for (int jj = 0; jj < n_kt; ++jj) {
+            const int j = kt0 + jj;  // absolute KV tile
+            const int b = jj & 1;
+            ok = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(bar(B_SFULL + 2 * t + b), (jj >> 1) & 1, p.err));
             if (!ok) break;
             tc_fence_after();
             float s[kKT];
@@ -350,7 +394,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 alpha = ex2(m_used - m_cand);
                 m_used = m_cand;
             }
-            const float neg_m = -m_used;
+            // a row whose keys in this range are all masked keeps m = -inf and p = 0
+            const float neg_m = m_used == -INFINITY ? 0.f : -m_used;
             float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
 #pragma unroll
             for (int i = 0; i < kKT; i += 4) {
@@ -365,9 +410,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             l_run = l_run * alpha + ((r0 + r1) + (r2 + r3));
 
-            if (j >= 1) {
-                // P_t(j-1) consumed and O_t(j-1) complete
-                ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (j - 1) & 1, p.err));
+            if (jj >= 1) {
+                // P_t(jj-1) consumed and O_t(jj-1) complete
+                ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (jj - 1) & 1, p.err));
                 if (!ok) break;
                 tc_fence_after();
                 if (__any_sync(0xffffffffu, need)) {
@@ -382,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_wait_st();
                 }
             }
-            if (j == n_kt - 1) {
+            if (j == n_kt_all - 1) {
                 // rows of the last page past the context may hold anything:
                 // zero them in V so that P = 0 times V stays 0.  Each tile's
                 // warpgroup does it before releasing its own P, so both P V
@@ -390,8 +435,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // zeros again)
                 const int keys_here = min(kKT, sq.ctx_len - first_key);
                 if (keys_here & (kPage - 1)) {
-                    const int s_idx = j % kNS;
-                    ok = __all_sync(0xffffffffu, mbar_wait(bar(B_VFULL + s_idx), (j / kNS) & 1, p.err));
+                    const int s_idx = jj % kNS;
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar(B_VFULL + s_idx), (jj / kNS) & 1, p.err));
                     if (!ok) break;
                     const int pg = keys_here / kPage, from = keys_here & (kPage - 1);
                     const int n = (kPage - from) * 8;  // 16-byte chunks per half
@@ -416,35 +461,91 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
 
         if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (n_kt - 1) & 1, p.err));
-        if (ok) {
-            tc_fence_after();
-            const float inv_l = 1.f / l_run;
-            const int64_t orow = static_cast<int64_t>(sq.q_start + t0 + r) * p.n_q_heads + h0 + t;
+        const int64_t orow = static_cast<int64_t>(sq.q_start + t0 + r) * p.n_q_heads + h0 + t;
+        const int nthr = hpc * 128;  // threads of the softmax warpgroups (named barrier 1)
+        if (n_splits == 1) {
+            if (ok) {
+                tc_fence_after();
+                const float inv_l = 1.f / l_run;
 #pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                float v[32];
-                tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
-                if (r < rows_valid) {
-                    if (p.out_fp32) {
-                        float4 *dst =
-                            reinterpret_cast<float4 *>(static_cast<float *>(p.out) + orow * kHeadDim + c4 * 32);
-#pragma unroll
-                        for (int i = 0; i < 8; ++i)
-                            dst[i] = make_float4(v[4 * i] * inv_l, v[4 * i + 1] * inv_l, v[4 * i + 2] * inv_l,
-                                                 v[4 * i + 3] * inv_l);
-                    } else {
-                        uint4 *dst = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.out) +
-                                                               orow * kHeadDim + c4 * 32);
-#pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            dst[i] = make_uint4(pack_bf16x2(v[8 * i] * inv_l, v[8 * i + 1] * inv_l),
-                                                pack_bf16x2(v[8 * i + 2] * inv_l, v[8 * i + 3] * inv_l),
-                                                pack_bf16x2(v[8 * i + 4] * inv_l, v[8 * i + 5] * inv_l),
-                                                pack_bf16x2(v[8 * i + 6] * inv_l, v[8 * i + 7] * inv_l));
-                    }
+                for (int c4 = 0; c4 < 4; ++c4) {
+                    float v[32];
+                    tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+                    if (r < rows_valid) store_row32(p, orow, c4, v, inv_l);
                 }
             }
         } else {
+            // split-KV: write this range's (m, l, O) for the row, then the last
+            // CTA of the tile merges every range:
+            //   o = sum_i 2^(m_i - M) o_i / sum_i 2^(m_i - M) l_i,  M = max_i m_i
+            const int split = static_cast<int>(wk.split & 0xFFFFu);
+            const int64_t prow = ((static_cast<int64_t>(wk.part + split) * slots + slot) * hpc + t) * kTileQ + r;
+            if (ok) {
+                tc_fence_after();
+                float4 *dst = reinterpret_cast<float4 *>(p.part_o + prow * kHeadDim);
+#pragma unroll
+                for (int c4 = 0; c4 < 4; ++c4) {
+                    float v[32];
+                    tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i)
+                        __stcg(dst + c4 * 8 + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+                }
+                __stcg(reinterpret_cast<float2 *>(p.part_ml + prow * 2), make_float2(m_used, l_run));
+            }
+            __threadfence();
+            const int any_fail = named_barrier_or(1, nthr, !ok);
+            int *s_last = reinterpret_cast<int *>(sg + kOffAbort + 4);
+            if (!any_fail) {
+                if (t == 0 && r == 0) {
+                    int *ticket = p.tickets + static_cast<int64_t>(wk.part) * slots + slot;
+                    const int prev = atomicAdd(ticket, 1);
+                    *s_last = (prev == n_splits - 1);
+                    if (prev == n_splits - 1) *ticket = 0;  // ready for the next call
+                }
+                named_barrier_sync(1, nthr);
+                if (*reinterpret_cast<volatile int *>(s_last)) {
+                    __threadfence();
+                    float M = -INFINITY;
+                    for (int i = 0; i < n_splits; ++i) {
+                        const int64_t q = ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
+                        M = fmaxf(M, __ldcg(p.part_ml + q * 2));
+                    }
+                    float L = 0.f;
+                    for (int i = 0; i < n_splits; ++i) {
+                        const int64_t q = ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
+                        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + q * 2));
+                        L += (ml.x == -INFINITY ? 0.f : ex2(ml.x - M)) * ml.y;
+                    }
+                    const float inv_l = 1.f / L;
+#pragma unroll 1
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        float acc[32];
+#pragma unroll
+                        for (int c = 0; c < 32; ++c) acc[c] = 0.f;
+                        for (int i = 0; i < n_splits; ++i) {
+                            const int64_t q =
+                                ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
+                            const float mi = __ldcg(p.part_ml + q * 2);
+                            const float f = mi == -INFINITY ? 0.f : ex2(mi - M);
+                            const float4 *src = reinterpret_cast<const float4 *>(p.part_o + q * kHeadDim + c4 * 32);
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                const float4 v = __ldcg(src + c);
+                                acc[4 * c] += f * v.x;
+                                acc[4 * c + 1] += f * v.y;
+                                acc[4 * c + 2] += f * v.z;
+                                acc[4 * c + 3] += f * v.w;
+                            }
+                        }
+                        if (r < rows_valid) store_row32(p, orow, c4, acc, inv_l);
+                    }
+                }
+            } else {
+                ok = false;
+            }
+        }
+        if (!ok) {
             *abort_flag = 1;
         }
       }
@@ -467,8 +568,8 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    if (p.n_tiles <= 0) return cudaSuccess;
-    const int grid = p.n_tiles * (p.n_q_heads / p.heads_per_cta);
+    if (p.n_work <= 0) return cudaSuccess;
+    const int grid = p.n_work * (p.n_q_heads / p.heads_per_cta);
     prefill_attn_kernel<<<grid, kThreads, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
     return cudaGetLastError();
 }

@@ -20,17 +20,31 @@ constexpr int kPageBytes = kPage * kRowBytes;  // one (block, kv-head) page: 4 K
 
 // ------------------------------------------------------------------ prefill
 // Rows with q_len > 1.  One CTA computes one 128-token query tile of
-// heads_per_cta q-heads of one kv-head against the tile's causal key range.
-constexpr int kTileQ = 128;      // query tokens per tile (tcgen05 M)
-constexpr int kTileK = 128;      // keys per KV tile (tcgen05 N of Q.K^T, K of P.V)
+// heads_per_cta q-heads of one kv-head over a range of its causal KV tiles.
+// Long ranges are split over several CTAs (split-KV); each split writes a
+// partial (m, l, O) and the last CTA of the tile merges them.
+constexpr int kTileQ = 128;            // query tokens per tile (tcgen05 M)
+constexpr int kPrefillKT = 64;         // keys per KV tile
 constexpr int kMaxPrefillSeqs = 128;
-constexpr int kMaxPrefillTiles = 1024;
+constexpr int kMaxPrefillWork = 1024;  // work items per launch
+// split-KV sizing: a step is cut into about this many CTAs, with at least
+// kPrefillMinSplitTiles KV tiles per CTA and at most kPrefillMaxSplits per tile
+constexpr int64_t kPrefillTargetCtas = 304;
+constexpr int kPrefillMinSplitTiles = 16;
+constexpr int kPrefillMaxSplits = 64;
 
 struct PrefillSeq {
     int32_t q_start;   // first row of the sequence in packed q / out
     int32_t q_len;
     int32_t ctx_len;
     int32_t table_row; // row of d_block_tables
+};
+
+struct PrefillWork {
+    uint32_t seq_qt;    // (launch-local sequence << 16) | q tile
+    uint32_t kt_range;  // (first KV tile << 16) | end KV tile (exclusive)
+    int32_t part;       // first partial slot of this tile's splits; -1: not split
+    uint32_t split;     // (number of splits << 16) | this split
 };
 
 struct PrefillParams {
@@ -41,14 +55,32 @@ struct PrefillParams {
     int32_t out_fp32;
     int32_t n_q_heads;
     int32_t n_kv_heads;
-    int32_t group;       // n_q_heads / n_kv_heads
+    int32_t group;          // n_q_heads / n_kv_heads
     int32_t heads_per_cta;  // 2 when the group has >= 2 heads, else 1
-    float scale_log2;    // scale * log2(e)
+    float scale_log2;       // scale * log2(e)
     int32_t *err;
-    int32_t n_tiles;     // tiles in this launch; grid = n_tiles * n_q_heads / heads_per_cta
-    uint32_t tiles[kMaxPrefillTiles];  // (seq << 16) | q_tile, heaviest first
+    float *part_o;          // [n_part, slots, heads_per_cta, 128 rows, 128]
+    float *part_ml;         // [n_part, slots, heads_per_cta, 128 rows, 2]
+    int32_t *tickets;       // [n_part, slots] (first slot of each split tile)
+    int32_t n_work;         // work items in this launch; grid = n_work * slots
+    PrefillWork work[kMaxPrefillWork];  // heaviest first
     PrefillSeq seqs[kMaxPrefillSeqs];
 };
+
+struct PrefillItem {
+    int32_t seq, qt, kt0, kt1, part, split, n_splits;
+};
+
+struct PrefillPlan {
+    std::vector<PrefillItem> items;  // sorted heaviest first
+    int64_t n_part = 0;
+    int32_t slots = 0, heads_per_cta = 1;
+    size_t o_bytes = 0, ml_bytes = 0, ticket_bytes = 0;
+    size_t total_bytes() const { return o_bytes + ml_bytes + ticket_bytes; }
+};
+
+PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                         int32_t n_kv_heads, bool allow_split);
 
 // ------------------------------------------------------------------ decode
 // Rows with q_len == 1.  One CTA handles one (row, kv-head, split): the
@@ -98,6 +130,10 @@ struct DecodePlan {
     size_t ml_bytes = 0, o_bytes = 0, counter_bytes = 0;
     size_t total_bytes() const { return ml_bytes + o_bytes + counter_bytes; }
 };
+
+// workspace the step needs without prefill splits (decode partials only)
+size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                          int32_t n_kv_heads);
 
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
                        int32_t n_kv_heads, int32_t num_sms);

@@ -86,5 +86,8 @@ def test_workspace_size_is_a_pure_function_of_lengths(ppas):
     a = ppas.ppas_attention_workspace_size([1, 1, 512], [25000, 25010, 3000], 16, 2)
     b = ppas.ppas_attention_workspace_size([1, 1, 512], [25000, 25010, 3000], 16, 2)
     assert a == b and a > 0 and a % 256 == 0
-    assert ppas.ppas_attention_workspace_size([512], [3000], 16, 2) == 0   # no decode rows
+    # a short chunk with no prefix: no decode rows and no split-KV ranges
+    assert ppas.ppas_attention_workspace_size([512], [512], 16, 2) == 0
+    # a chunk over a long prefix is split over its KV range: partials need room
+    assert ppas.ppas_attention_workspace_size([512], [24000], 16, 2) > 0
     assert ppas.ppas_attention_workspace_size([], [], 16, 2) == 0

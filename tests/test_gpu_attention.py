@@ -35,6 +35,7 @@ SMALL_SHAPES = [
     wl.StepShape([1, 37, 1, 300], [40, 37, 129, 1000]),           # mixed, unaligned prefixes
     wl.StepShape([2, 257, 129], [2, 700, 129 + 384]),             # several q tiles, prefix % 128 != 0
     wl.StepShape([1] * 5 + [64], [4000, 3999, 2050, 16, 1, 5000]),  # decodes with splits
+    wl.StepShape([1, 200], [5000, 6000]),                        # chunk tiles split over their KV range
 ]
 
 
@@ -232,3 +233,25 @@ def test_full_size_sampled_rows(ppas, name, geo, mk):
     rows = sample_rows(shape, geo.n_q_heads, 96, seed=1)
     got = o[[r for r, _ in rows], [h for _, h in rows]]
     assert_close(got, oracle_rows(c, rows), name)
+
+
+def test_split_kv_and_unsplit_fallback_agree(ppas):
+    """A chunk over a long prefix runs split over its KV range (partials merged
+    by the last CTA); with a workspace too small for the partials the same
+    step runs unsplit.  Both match the oracle."""
+    geo = QWEN
+    shape = wl.StepShape([1, 300, 130], [9000, 12000, 7000])
+    c = device_case(geo, shape, seed=21, nan_fill=True)
+    want = oracle_full(c)
+    full = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads)
+    outs = []
+    for ws_bytes in (full, 1 << 20):
+        out = torch.empty((shape.total_q, geo.n_q_heads, geo.head_dim), dtype=torch.float32, device="cuda")
+        ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+        ppas.ppas_attention_step(c.q, c.k_cache, c.v_cache, c.num_blocks, c.tables, c.width, shape.q_lens,
+                                 shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads, geo.head_dim, c.scale, out, True,
+                                 ws, ws_bytes)
+        torch.cuda.synchronize()
+        assert_close(host64(out), want, f"workspace {ws_bytes}")
+        outs.append(out)
+    assert full > 1 << 20

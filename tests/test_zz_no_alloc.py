@@ -28,7 +28,11 @@ def ppas():
 def test_noalloc_matches_workspace_entry_point_twice(ppas):
     geo = wl.QWEN25_3B
     shape = wl.high_pressure_step(0)          # 8 decode rows of ~25k context (several splits) + 4 chunks
-    need = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads)
+    # the decode rows' split scratch fits the fixed array; the prefill chunks
+    # then run without KV splits (their partials would not fit)
+    dec = [i for i, q in enumerate(shape.q_lens) if q == 1]
+    need = ppas.ppas_attention_workspace_size([1] * len(dec), [shape.ctx_lens[i] for i in dec], geo.n_q_heads,
+                                              geo.n_kv_heads)
     assert 0 < need <= ppas.PPAS_NOALLOC_SCRATCH_BYTES
     c = device_case(geo, shape, seed=5)
     want = run_step(ppas, c, out_fp32=True)
