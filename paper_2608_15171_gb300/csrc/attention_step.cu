@@ -15,9 +15,9 @@ namespace ppas {
 namespace {
 
 // Decode rows are split so that one step launches about this many CTAs
-// (two per SM on a 152-SM GB300).  A fixed number keeps the workspace size a
+// (one per SM on a 152-SM GB300).  A fixed number keeps the workspace size a
 // pure function of the step's lengths.
-constexpr int64_t kDecodeTargetCtas = 304;
+constexpr int64_t kDecodeTargetCtas = 152;
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -84,21 +84,26 @@ bool encode_q_map(CUtensorMap *map, const void *q, int32_t total_q, int32_t n_q_
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
                        int32_t n_kv_heads, int32_t /*num_sms*/) {
     DecodePlan d;
-    int64_t total_pages = 0;
+    int64_t total_pages = 0;  // over (row, kv-head) pairs
     for (int32_t s = 0; s < n_seqs; ++s)
         if (q_lens[s] == 1) {
             d.rows.push_back(s);
             total_pages += static_cast<int64_t>((ctx_lens[s] + kPage - 1) / kPage) * n_kv_heads;
         }
     if (d.rows.empty()) return d;
-    int64_t pps = (total_pages + kDecodeTargetCtas - 1) / kDecodeTargetCtas;
-    pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
-    pps = (pps + kDecodeWarps - 1) / kDecodeWarps * kDecodeWarps;
-    d.pages_per_split = static_cast<int32_t>(pps);
+    // each (row, kv-head) gets a share of about kDecodeTargetCtas CTAs in
+    // proportion to its pages, so one step stays within one wave
     for (int32_t s : d.rows) {
         const int64_t pages = (ctx_lens[s] + kPage - 1) / kPage;
+        int64_t share = kDecodeTargetCtas * pages * n_kv_heads / total_pages / n_kv_heads;
+        share = std::max<int64_t>(share, 1);
+        int64_t pps = (pages + share - 1) / share;
+        pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
+        pps = (pps + kDecodeWarps - 1) / kDecodeWarps * kDecodeWarps;
+        pps = std::min<int64_t>(pps, kDecodeMaxPagesPerSplit);
         const int32_t ns = static_cast<int32_t>((pages + pps - 1) / pps);
         d.n_splits.push_back(ns);
+        d.pages_per_split.push_back(static_cast<int32_t>(pps));
         d.n_part += ns;
         d.n_ctas += static_cast<int64_t>(ns) * n_kv_heads;
     }
@@ -298,7 +303,6 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         dprm.n_kv_heads = n_kv_heads;
         dprm.group = g;
         dprm.scale_log2 = scale_log2;
-        dprm.pages_per_split = dp.pages_per_split;
         dprm.part_ml = part_ml;
         dprm.part_o = part_o;
         dprm.err = d_err_flag;
@@ -315,6 +319,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
                 r.ctx_len = h_ctx_lens[s];
                 r.table_row = s;
                 r.n_splits = dp.n_splits[i];
+                r.pages_per_split = dp.pages_per_split[i];
                 r.cta_base = cta;
                 r.part_base = part_base;
                 cta += r.n_splits * n_kv_heads;

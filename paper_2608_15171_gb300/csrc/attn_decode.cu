@@ -3,11 +3,13 @@
 // A decode row is bandwidth-bound: every K/V byte is read once and used by
 // the group's q-heads only.  One CTA takes one (row, kv-head, split): its
 // pages are fetched by TMA (two 16x64 boxes per page and matrix, 128-byte
-// swizzle) into a 4-stage ring per warp; each warp computes
+// swizzle) into a 3-stage ring per warp (eight warps, so eight threads issue
+// copies; one issuing thread alone moves only ~7 B/clk); the split's page ids
+// are staged in shared memory first.  Each warp computes
 //   S^T[heads x 16 keys] = Q[heads x 128] . K_page^T     (mma.sync m16n8k16)
 //   online softmax per head (fp32, exp2 domain)
 //   O[heads x 128] += P[heads x 16 keys] . V_page         (mma.sync m16n8k16)
-// with the group's q-heads as the MMA rows (rows >= group are zero).  The four
+// with the group's q-heads as the MMA rows (rows >= group are zero).  The
 // warps merge their (m, l, O) in shared memory; with several splits the
 // partial goes to the workspace and the last CTA of the (row, kv-head) to
 // finish merges all splits:
@@ -25,7 +27,9 @@ constexpr uint32_t kStageBytes = 4 * kBox;          // K lo, K hi, V lo, V hi
 constexpr uint32_t kRingBytes = kDecodeStages * kStageBytes;
 constexpr uint32_t kOffBar = kDecodeWarps * kRingBytes;
 constexpr uint32_t kOffFlag = kOffBar + kDecodeWarps * kDecodeStages * 8;
-constexpr uint32_t kSmemBytes = kOffFlag + 16 + 1024;
+constexpr uint32_t kOffIds = kOffFlag + 16;   // page ids of this split
+constexpr uint32_t kSmemBytes = kOffIds + kDecodeMaxPagesPerSplit * 4 + 1024;
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 // merge scratch (aliases the rings once every warp is done)
 constexpr int kMaxGroup = 8;
 static_assert(kDecodeWarps * kMaxGroup * (2 + kHeadDim) * 4 <= static_cast<int>(kOffBar), "merge scratch");
@@ -77,25 +81,28 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     const int kvh = local / row.n_splits, sp = local % row.n_splits;
     const int g = p.group;
     const int n_pages = (row.ctx_len + kPage - 1) / kPage;
-    const int pg0 = sp * p.pages_per_split;
-    const int pg1 = min(pg0 + p.pages_per_split, n_pages);
+    const int pg0 = sp * row.pages_per_split;
+    const int pg1 = min(pg0 + row.pages_per_split, n_pages);
     const int my_count = max(0, (pg1 - pg0 - warp + kDecodeWarps - 1) / kDecodeWarps);
     const int32_t *table = p.block_tables + static_cast<int64_t>(row.table_row) * p.table_stride;
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sg + kOffFlag);
 
     const uint32_t ring = sb + warp * kRingBytes;
     auto bar = [&](int st) { return sb + kOffBar + (warp * kDecodeStages + st) * 8u; };
+    int32_t *ids = reinterpret_cast<int32_t *>(sg + kOffIds);
     if (lane == 0) {
         for (int st = 0; st < kDecodeStages; ++st) mbar_init(bar(st), 1);
         fence_mbar_init();
     }
     if (tid == 0) *abort_flag = 0;
+    // the split's page ids, loaded once by every thread in parallel
+    for (int i = tid; i < pg1 - pg0; i += blockDim.x) ids[i] = __ldg(table + pg0 + i);
     __syncthreads();
 
     auto issue = [&](int i) {
         const int st = i % kDecodeStages;
         const int pg = pg0 + warp + kDecodeWarps * i;
-        int blk = __ldg(table + pg);
+        int blk = ids[pg - pg0];
         if (blk < 0 || blk >= p.num_blocks) {
             report_error(p.err, PPAS_DEVERR_BAD_INDEX);
             blk = 0;
@@ -225,8 +232,11 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     __syncthreads();
     if (*abort_flag) return;
 
-    const int t = tid;  // head-dim column merged by this thread
-    for (int hh = 0; hh < g; ++hh) {
+    // thread -> (head-dim column, first head); the CTA's threads cover
+    // blockDim.x / 128 heads at a time
+    const int t = tid & (kHeadDim - 1);
+    const int hstep = blockDim.x / kHeadDim;
+    for (int hh = tid / kHeadDim; hh < g; hh += hstep) {
         float M = -INFINITY;
 #pragma unroll
         for (int w = 0; w < kDecodeWarps; ++w) M = fmaxf(M, cm[w * kMaxGroup + hh]);
@@ -266,7 +276,7 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    for (int hh = 0; hh < g; ++hh) {
+    for (int hh = tid / kHeadDim; hh < g; hh += hstep) {
         const int head = kvh * g + hh;
         float M = -INFINITY;
         for (int s = 0; s < row.n_splits; ++s)

@@ -86,8 +86,9 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
 // Rows with q_len == 1.  One CTA handles one (row, kv-head, split): the
 // split's pages are spread over the CTA's warps; partial (m, l, o) go to the
 // workspace and the last CTA of a (row, kv-head) combines them.
-constexpr int kDecodeWarps = 4;
-constexpr int kDecodeStages = 4;       // pages in flight per warp
+constexpr int kDecodeWarps = 8;        // each warp streams its own pages (8 TMA issuers per SM)
+constexpr int kDecodeStages = 3;       // pages in flight per warp
+constexpr int kDecodeMaxPagesPerSplit = 1024;  // page ids of a split are staged in shared memory
 constexpr int kMaxDecodeRows = 256;
 constexpr int kDecodeMinPagesPerSplit = 16;
 
@@ -96,6 +97,7 @@ struct DecodeRow {
     int32_t ctx_len;
     int32_t table_row;
     int32_t n_splits;
+    int32_t pages_per_split;
     int32_t cta_base;    // first CTA of this row (all kv-heads)
     int32_t part_base;   // first partial slot (units of splits) of this row
 };
@@ -111,7 +113,6 @@ struct DecodeParams {
     int32_t n_kv_heads;
     int32_t group;
     float scale_log2;
-    int32_t pages_per_split;
     float *part_ml;      // [n_part, n_q_heads, 2]   (m, l)
     float *part_o;       // [n_part, n_q_heads, 128] unnormalised
     int32_t *counters;   // [n_rows, n_kv_heads]
@@ -122,9 +123,9 @@ struct DecodeParams {
 };
 
 struct DecodePlan {
-    int32_t pages_per_split = 0;
     std::vector<int32_t> rows;       // indices of q_len == 1 rows
     std::vector<int32_t> n_splits;   // per decode row
+    std::vector<int32_t> pages_per_split;  // per decode row
     int64_t n_part = 0;              // sum of splits
     int64_t n_ctas = 0;
     size_t ml_bytes = 0, o_bytes = 0, counter_bytes = 0;
