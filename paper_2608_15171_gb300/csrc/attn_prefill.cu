@@ -1,23 +1,29 @@
 // Prefill-chunk attention on the 5th-generation tensor cores (tcgen05).
 //
 // One CTA computes O for one 128-token query tile of two q-heads of the same
-// kv-head (one head when the group size is 1); both Q tiles share every K/V
-// tile it loads.  Warp roles (512 threads, four warpgroups):
-//   warps 0-3   TMA producers: warp w owns ring stage w and fetches the
-//               64-key K and V tiles j = w, w+4, ... (four 16-token pages
-//               each, through the block table); warp 0 also loads Q.  One
+// kv-head (one head when the group size is 1) over a range of 128-key KV
+// tiles; both Q tiles share every K/V tile it loads.  Per Q tile t the work
+// is a chain  S_t = Q_t K^T  ->  softmax  ->  P_t (bf16, written over S_t in
+// TMEM)  ->  O_t += P_t V, and the two tiles' chains interleave on the
+// tensor core.  Warp roles (512 threads, four warpgroups):
+//   warps 0-3   TMA producers: warps 0/1 fetch pages 0-3 / 4-7 of each K
+//               tile (3-stage ring), warps 2/3 those of each V tile (2
+//               stages), through the block table; warp 0 also loads Q.  One
 //               issuing thread moves only ~7 B/clk of small TMA boxes on
-//               GB300, so the ring is filled by four threads in parallel.
-//   warps 4, 5  MMA issuers, one thread per Q tile: S_t = Q_t K^T into TMEM
-//               (double buffered, one KV tile ahead), then O_t += P_t V
-//   warps 8-11  softmax for tile 0, warps 12-15 softmax for tile 1: each
-//               thread owns one query row (its TMEM lane), loads its S row,
-//               masks by absolute position, runs the online softmax in fp32
-//               (exp2 domain), writes P (bf16) to shared memory
+//               GB300, so every tile is fetched by two threads.
+//   warps 4, 5  MMA issuers, one thread per Q tile: S_t = Q_t K^T (A = Q in
+//               shared memory) and O_t += P_t V (A = P in TMEM); Q K^T for the
+//               next tile is issued once P V has consumed P.
+//   warps 8-11  softmax for tile 0, warps 12-15 for tile 1: each thread owns
+//               one query row (its TMEM lane), loads its S row, masks by
+//               absolute position, runs the online softmax in fp32 (exp2
+//               domain) and stores P back to TMEM
 // Registers move from the producer/MMA warpgroups to the softmax warpgroups
 // with setmaxnreg.  The running max is only raised (and O rescaled in TMEM)
 // when it grows by more than 2^8; until then the stale max keeps every
 // exponent <= 2^8, and the final O / l is exact either way.
+// Long KV ranges may be split over several CTAs (split-KV): each writes its
+// partial (m, l, O) and the last one of the tile merges them.
 #include <math.h>
 
 #include "ppas_device.cuh"
@@ -26,46 +32,42 @@
 namespace ppas {
 namespace {
 
-constexpr int kKT = kPrefillKT;            // keys per KV tile
-constexpr int kNS = 4;                     // KV ring depth
-constexpr int kPagesPerTile = kKT / kPage; // 4
-constexpr uint32_t kBox = 2048;            // one TMA box: 16 rows x 128 B
-constexpr uint32_t kQHalf = 16384;         // 128 rows x 128 B (64 columns)
-constexpr uint32_t kQBytes = 2 * kQHalf;
-constexpr uint32_t kKVHalf = 8192;         // 64 rows x 128 B
-constexpr uint32_t kKVBytes = 2 * kKVHalf;
-constexpr uint32_t kPBytes = 16384;        // 128 rows x 64 keys bf16
+constexpr int kKT = kPrefillKT;              // keys per KV tile (128)
+constexpr int kPagesPerTile = kKT / kPage;   // 8
+constexpr int kNK = 3;                       // K ring depth
+constexpr int kNV = 2;                       // V ring depth
+constexpr uint32_t kBox = 2048;              // one TMA box: 16 rows x 128 B
+constexpr uint32_t kHalf = 16384;            // 128 rows x 128 B (64 columns)
+constexpr uint32_t kTileBytes = 2 * kHalf;   // a Q, K or V tile: 128 rows x 256 B
 
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = kOffQ + 2 * kQBytes;
-constexpr uint32_t kOffV = kOffK + kNS * kKVBytes;
-constexpr uint32_t kOffP = kOffV + kNS * kKVBytes;
-constexpr uint32_t kOffBar = kOffP + 2 * kPBytes;
+constexpr uint32_t kOffK = kOffQ + 2 * kTileBytes;
+constexpr uint32_t kOffV = kOffK + kNK * kTileBytes;
+constexpr uint32_t kOffBar = kOffV + kNV * kTileBytes;
 enum : int {
     B_Q = 0,
     B_KFULL = 1,
-    B_KEMPTY = B_KFULL + kNS,
-    B_VFULL = B_KEMPTY + kNS,
-    B_VEMPTY = B_VFULL + kNS,
-    B_SFULL = B_VEMPTY + kNS,  // [tile][buffer]
-    B_SFREE = B_SFULL + 4,     // [tile][buffer]
-    B_PFULL = B_SFREE + 4,     // [tile]
+    B_KEMPTY = B_KFULL + kNK,
+    B_VFULL = B_KEMPTY + kNK,
+    B_VEMPTY = B_VFULL + kNV,
+    B_SFULL = B_VEMPTY + kNV,  // [tile]
+    B_PFULL = B_SFULL + 2,     // [tile]
     B_ODONE = B_PFULL + 2,     // [tile]
-    B_DRAIN = B_ODONE + 2,
+    B_TURN = B_ODONE + 2,      // [tile]: the softmax warpgroups take turns
+    B_DRAIN = B_TURN + 2,
     B_COUNT = B_DRAIN + 1
 };
 constexpr uint32_t kOffTmem = kOffBar + B_COUNT * 8;
 constexpr uint32_t kOffAbort = kOffTmem + 4;
-static_assert(kOffAbort + 4 <= kOffBar + 256, "barrier area");
+constexpr uint32_t kOffLast = kOffAbort + 4;
+static_assert(kOffLast + 4 <= kOffBar + 256, "barrier area");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 232448, "shared memory per CTA");
-constexpr uint32_t kTmemCols = 512;  // S[2 tiles][2 buffers] x 64 cols, O[2 tiles] x 128 cols
-constexpr uint32_t kColO = 256;
+constexpr uint32_t kTmemCols = 512;  // tile t: S/P at t*256, O at t*256 + 128
 constexpr float kRescaleThreshold = 8.0f;  // log2 units
 constexpr int kThreads = 512;
-constexpr int kProducerWarps = kNS;        // warps 0..3, one per ring stage
-constexpr int kMmaWarp = 4;                // warps 4..7 form the MMA warpgroup
-constexpr int kSoftmaxWarp0 = 8;           // warps 8..11 tile 0, 12..15 tile 1
+constexpr int kMmaWarp = 4;       // warps 4..7 form the MMA warpgroup
+constexpr int kSoftmaxWarp0 = 8;  // warps 8..11 tile 0, 12..15 tile 1
 // register split: 8 warps x 56 + 8 warps x 200 = 512 threads x 128 at launch
 constexpr int kRegsSmall = 56;
 constexpr int kRegsLarge = 200;
@@ -125,6 +127,31 @@ __device__ __forceinline__ void tmem_st32_f(uint32_t taddr, const float (&v)[32]
     tmem_st32(taddr, r);
 }
 
+// two fp32 lanes at once (Blackwell packed FP32 pipe)
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return r;
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    float2 r;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
 __device__ __forceinline__ void named_barrier_sync(int id, int n) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
@@ -162,6 +189,7 @@ __device__ __forceinline__ void store_row32(const PrefillParams &p, int64_t orow
     }
 }
 
+
 }  // namespace
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -184,11 +212,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int prefix = sq.ctx_len - sq.q_len;
     const int kvh = h0 / p.group;
     const int last_pos = prefix + t0 + rows_valid - 1;
-    const int n_kt_all = last_pos / kKT + 1;           // KV tiles of the whole causal range
+    const int n_kt_all = last_pos / kKT + 1;              // KV tiles of the whole causal range
     const int kt0 = static_cast<int>(wk.kt_range >> 16);  // this CTA's range [kt0, kt0 + n_kt)
     const int n_kt = static_cast<int>(wk.kt_range & 0xFFFFu) - kt0;
     const int n_splits = static_cast<int>(wk.split >> 16);
     const int32_t *table = p.block_tables + static_cast<int64_t>(sq.table_row) * p.table_stride;
+    // pages of KV tile j that hold at least one context key
+    auto pages_in = [&](int j) { return min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage); };
 
     auto bar = [&](int i) { return sb + kOffBar + 8u * static_cast<uint32_t>(i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sg + kOffAbort);
@@ -199,19 +229,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (tid == 0) {
         mbar_init(bar(B_Q), 1);
-        for (int s = 0; s < kNS; ++s) {
-            mbar_init(bar(B_KFULL + s), 1);
-            mbar_init(bar(B_KEMPTY + s), hpc);  // one release per tile's MMA thread
-            mbar_init(bar(B_VFULL + s), 1);
+        for (int s = 0; s < kNK; ++s) {
+            mbar_init(bar(B_KFULL + s), 2);      // two producer threads per tile
+            mbar_init(bar(B_KEMPTY + s), hpc);   // one release per tile's MMA thread
+        }
+        for (int s = 0; s < kNV; ++s) {
+            mbar_init(bar(B_VFULL + s), 2);
             mbar_init(bar(B_VEMPTY + s), hpc);
         }
-        for (int i = 0; i < 4; ++i) {
-            mbar_init(bar(B_SFULL + i), 1);
-            mbar_init(bar(B_SFREE + i), 4);
-        }
         for (int t = 0; t < 2; ++t) {
+            mbar_init(bar(B_SFULL + t), 1);
             mbar_init(bar(B_PFULL + t), 4);
             mbar_init(bar(B_ODONE + t), 1);
+            mbar_init(bar(B_TURN + t), 4);
         }
         mbar_init(bar(B_DRAIN), hpc);
         *abort_flag = 0;
@@ -225,121 +255,108 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sg + kOffTmem);
 
-    if (warp < kProducerWarps) {
+    if (warp < 4) {
         // ------------------------------------------------------------ TMA producers
         asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsSmall));
         if (lane == 0) {
             if (warp == 0) {
-                mbar_expect_tx(bar(B_Q), static_cast<uint32_t>(hpc) * kQBytes);
+                mbar_expect_tx(bar(B_Q), static_cast<uint32_t>(hpc) * kTileBytes);
                 const int qrow = sq.q_start + t0;
                 for (int t = 0; t < hpc; ++t) {
-                    tma_load_3d(sb + kOffQ + t * kQBytes, &tm_q, 0, h0 + t, qrow, bar(B_Q));
-                    tma_load_3d(sb + kOffQ + t * kQBytes + kQHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
+                    tma_load_3d(sb + kOffQ + t * kTileBytes, &tm_q, 0, h0 + t, qrow, bar(B_Q));
+                    tma_load_3d(sb + kOffQ + t * kTileBytes + kHalf, &tm_q, 64, h0 + t, qrow, bar(B_Q));
                 }
             }
-            const int s = warp;  // this warp's ring stage: local tiles jj = s, s + kNS, ...
-            const uint32_t dk = sb + kOffK + s * kKVBytes, dv = sb + kOffV + s * kKVBytes;
+            const bool is_v = warp >= 2;
+            const int pg_lo = (warp & 1) * (kPagesPerTile / 2);  // this thread's pages of each tile
+            const int ns = is_v ? kNV : kNK;
+            const CUtensorMap *tm = is_v ? &tm_v : &tm_k;
+            const uint32_t ring = sb + (is_v ? kOffV : kOffK);
+            const int full0 = is_v ? B_VFULL : B_KFULL, empty0 = is_v ? B_VEMPTY : B_KEMPTY;
             // page ids of the next tile are loaded while the current one is issued
-            auto load_ids = [&](int jj, int (&ids)[kPagesPerTile]) {
+            int ids[kPagesPerTile / 2];
+            auto load_ids = [&](int jj) {
                 const int j = kt0 + jj;
-                const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
+                const int np = jj < n_kt ? pages_in(j) : 0;
 #pragma unroll
-                for (int pg = 0; pg < kPagesPerTile; ++pg)
-                    ids[pg] = (jj < n_kt && pg < n_pages) ? __ldg(table + j * kPagesPerTile + pg) : 0;
+                for (int i = 0; i < kPagesPerTile / 2; ++i)
+                    ids[i] = (pg_lo + i < np) ? __ldg(table + j * kPagesPerTile + pg_lo + i) : 0;
             };
-            int ids[kPagesPerTile];
-            load_ids(s, ids);
-            for (int jj = s; jj < n_kt; jj += kNS) {
+            load_ids(0);
+            for (int jj = 0; jj < n_kt; ++jj) {
                 const int j = kt0 + jj;
-                const uint32_t ph = (jj / kNS) & 1;
-                const int n_pages = min(kPagesPerTile, (sq.ctx_len - j * kKT + kPage - 1) / kPage);
-                int rows[kPagesPerTile];
+                const int s = jj % ns;
+                const int np = max(0, min(kPagesPerTile / 2, pages_in(j) - pg_lo));
+                int rows[kPagesPerTile / 2];
 #pragma unroll
-                for (int pg = 0; pg < kPagesPerTile; ++pg) {
-                    int blk = ids[pg];
-                    if (pg < n_pages && (blk < 0 || blk >= p.num_blocks)) {
+                for (int i = 0; i < kPagesPerTile / 2; ++i) {
+                    int blk = ids[i];
+                    if (i < np && (blk < 0 || blk >= p.num_blocks)) {
                         report_error(p.err, PPAS_DEVERR_BAD_INDEX);
                         blk = 0;  // keep the barrier's byte count consistent
                     }
-                    rows[pg] = (blk * p.n_kv_heads + kvh) * kPage;
+                    rows[i] = (blk * p.n_kv_heads + kvh) * kPage;
                 }
-                load_ids(jj + kNS, ids);
-                if (jj >= kNS && !mbar_wait(bar(B_KEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
-                mbar_expect_tx(bar(B_KFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
-                for (int pg = 0; pg < n_pages; ++pg) {
-                    tma_load_2d(dk + pg * kBox, &tm_k, 0, rows[pg], bar(B_KFULL + s));
-                    tma_load_2d(dk + kKVHalf + pg * kBox, &tm_k, 64, rows[pg], bar(B_KFULL + s));
+                load_ids(jj + 1);
+                if (jj >= ns && !mbar_wait(bar(empty0 + s), ((jj / ns) & 1) ^ 1, p.err)) {
+                    *abort_flag = 1;
+                    break;
                 }
-                if (jj >= kNS && !mbar_wait(bar(B_VEMPTY + s), ph ^ 1, p.err)) { *abort_flag = 1; break; }
-                mbar_expect_tx(bar(B_VFULL + s), static_cast<uint32_t>(n_pages) * 2 * kBox);
-                for (int pg = 0; pg < n_pages; ++pg) {
-                    tma_load_2d(dv + pg * kBox, &tm_v, 0, rows[pg], bar(B_VFULL + s));
-                    tma_load_2d(dv + kKVHalf + pg * kBox, &tm_v, 64, rows[pg], bar(B_VFULL + s));
+                const uint32_t b = bar(full0 + s);
+                mbar_expect_tx(b, static_cast<uint32_t>(np) * 2 * kBox);
+                const uint32_t dst = ring + s * kTileBytes + pg_lo * kBox;
+                for (int i = 0; i < np; ++i) {
+                    tma_load_2d(dst + i * kBox, tm, 0, rows[i], b);
+                    tma_load_2d(dst + kHalf + i * kBox, tm, 64, rows[i], b);
                 }
             }
         }
     } else if (warp < kSoftmaxWarp0) {
         // ------------------------------------------------------------ MMA issuers
-        // lane 0 of warp kMmaWarp + t issues every MMA of Q tile t; the two
-        // threads share only the K/V stages, which each releases once
         asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsSmall));
         const int t = warp - kMmaWarp;
         if (t < hpc && lane == 0) {
             bool ok = mbar_wait(bar(B_Q), 0, p.err);
-            tc_fence_after();
             // descriptors are built once; advancing one operand by b bytes
             // adds b >> 4 to the start-address field (no carry: < 256 KB)
-            const uint64_t dq = smem_desc_sw128(sb + kOffQ + t * kQBytes, 16, 1024);
+            const uint64_t dq = smem_desc_sw128(sb + kOffQ + t * kTileBytes, 16, 1024);
             const uint64_t dk0 = smem_desc_sw128(sb + kOffK, 16, 1024);
-            const uint64_t dv0 = smem_desc_sw128(sb + kOffV, kKVHalf, 1024);
-            const uint64_t dp = smem_desc_sw128(sb + kOffP + t * kPBytes, 16, 1024);
-            const uint32_t d_s = tmem + t * 128, d_o = tmem + kColO + t * 128;
-            // S_t(jj) = Q_t K(kt0 + jj)^T into S buffer jj % 2 of this tile
-            auto issue_qk = [&](int jj) -> bool {
-                const int s = jj % kNS, b = jj & 1;
-                if (!mbar_wait(bar(B_KFULL + s), (jj / kNS) & 1, p.err)) return false;
-                // the softmax has read S_t(jj-2) out of this buffer
-                if (jj >= 2 && !mbar_wait(bar(B_SFREE + 2 * t + b), ((jj >> 1) - 1) & 1, p.err)) return false;
+            const uint64_t dv0 = smem_desc_sw128(sb + kOffV, kHalf, 1024);
+            const uint32_t d_s = tmem + t * 256, d_o = tmem + t * 256 + 128;
+            for (int jj = 0; ok && jj < n_kt; ++jj) {
+                const int j = kt0 + jj;
+                // ---- S_t = Q_t K(j)^T, once P V (jj-1) has read P out of S's columns
+                const int sk = jj % kNK;
+                if (!mbar_wait(bar(B_KFULL + sk), (jj / kNK) & 1, p.err)) { ok = false; break; }
+                if (jj >= 1 && !mbar_wait(bar(B_ODONE + t), (jj - 1) & 1, p.err)) { ok = false; break; }
                 tc_fence_after();
-                const uint64_t dk = dk0 + ((s * kKVBytes) >> 4);
+                const uint64_t dk = dk0 + ((sk * kTileBytes) >> 4);
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
-                    const uint32_t qo = (kk >> 2) * kQHalf + (kk & 3) * 32;
-                    const uint32_t ko = (kk >> 2) * kKVHalf + (kk & 3) * 32;
-                    umma_bf16(d_s + b * kKT, dq + (qo >> 4), dk + (ko >> 4), kIdescQK, kk > 0 ? 1u : 0u);
+                    const uint32_t o = (kk >> 2) * kHalf + (kk & 3) * 32;
+                    umma_bf16(d_s, dq + (o >> 4), dk + (o >> 4), kIdescQK, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(bar(B_SFULL + 2 * t + b));
-                umma_commit(bar(B_KEMPTY + s));
-                return true;
-            };
-            // O_t += P_t(i) V(kt0 + i)
-            auto issue_pv = [&](int i) -> bool {
-                const int s = i % kNS;
-                if (!mbar_wait(bar(B_VFULL + s), (i / kNS) & 1, p.err)) return false;
-                if (!mbar_wait(bar(B_PFULL + t), i & 1, p.err)) return false;
+                umma_commit(bar(B_SFULL + t));
+                umma_commit(bar(B_KEMPTY + sk));
+                // ---- O_t += P_t V(j), P_t from TMEM
+                const int sv = jj % kNV;
+                if (!mbar_wait(bar(B_VFULL + sv), (jj / kNV) & 1, p.err)) { ok = false; break; }
+                if (!mbar_wait(bar(B_PFULL + t), jj & 1, p.err)) { ok = false; break; }
                 tc_fence_after();
-                const int chunks = min(kPagesPerTile, (sq.ctx_len - (kt0 + i) * kKT + kPage - 1) / kPage);
-                const uint64_t dv = dv0 + ((s * kKVBytes) >> 4);
+                const uint64_t dv = dv0 + ((sv * kTileBytes) >> 4);
+                const int chunks = pages_in(j);
                 if (chunks == kPagesPerTile) {
 #pragma unroll
                     for (int kk = 0; kk < kPagesPerTile; ++kk)
-                        umma_bf16(d_o, dp + ((kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescPV,
-                                  (i > 0 || kk > 0) ? 1u : 0u);
+                        umma_bf16_ts(d_o, d_s + kk * 8, dv + ((kk * 2048) >> 4), kIdescPV,
+                                     (jj > 0 || kk > 0) ? 1u : 0u);
                 } else {
                     for (int kk = 0; kk < chunks; ++kk)
-                        umma_bf16(d_o, dp + ((kk * 32) >> 4), dv + ((kk * 2048) >> 4), kIdescPV,
-                                  (i > 0 || kk > 0) ? 1u : 0u);
+                        umma_bf16_ts(d_o, d_s + kk * 8, dv + ((kk * 2048) >> 4), kIdescPV,
+                                     (jj > 0 || kk > 0) ? 1u : 0u);
                 }
                 umma_commit(bar(B_ODONE + t));
-                umma_commit(bar(B_VEMPTY + s));
-                return true;
-            };
-            // Q K^T runs one KV tile ahead of P V, so the next S is ready when
-            // the softmax warpgroup finishes the current one
-            if (ok) ok = issue_qk(0);
-            for (int j = 0; ok && j < n_kt; ++j) {
-                if (j + 1 < n_kt && !issue_qk(j + 1)) { ok = false; break; }
-                if (!issue_pv(j)) ok = false;
+                umma_commit(bar(B_VEMPTY + sv));
             }
             if (!ok) *abort_flag = 1;
             // every MMA issued so far completes before TMEM is released
@@ -356,23 +373,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pos = min(prefix + t0 + r, sq.ctx_len - 1);  // last key this row may see
         const int min_pos = prefix + t0;
         const uint32_t t_lane = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+        const uint32_t t_s = t_lane + t * 256, t_o = t_lane + t * 256 + 128;
         const float sl2 = p.scale_log2;
         float m_used = -INFINITY, l_run = 0.f;
         bool ok = true;
-        uint8_t *prow = sg + kOffP + t * kPBytes + (r >> 3) * 1024 + (r & 7) * 128;
 
         for (int jj = 0; jj < n_kt; ++jj) {
             const int j = kt0 + jj;  // absolute KV tile
-            const int b = jj & 1;
-            ok = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(bar(B_SFULL + 2 * t + b), (jj >> 1) & 1, p.err));
+            // S_t(jj) ready; it was issued after P V (jj-1) completed, so O_t is stable
+            ok = __all_sync(0xffffffffu, !*abort_flag && mbar_wait(bar(B_SFULL + t), jj & 1, p.err));
+            // the two tiles' softmax phases alternate (tile 0 first), so one
+            // tile's softmax overlaps the other tile's MMAs instead of both
+            // competing for the exponential and FP32 pipes at once
+            if (ok && hpc == 2 && (t == 1 || jj > 0))
+                ok = __all_sync(0xffffffffu, mbar_wait(bar(B_TURN + t), (t == 0 ? jj - 1 : jj) & 1, p.err));
             if (!ok) break;
             tc_fence_after();
             float s[kKT];
-            tmem_ld64_sync(t_lane + t * 128 + b * kKT, s);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(B_SFREE + 2 * t + b));
-
+            {
+                float h[64];
+                tmem_ld64_sync(t_s, h);
+#pragma unroll
+                for (int i = 0; i < 64; ++i) s[i] = h[i];
+                tmem_ld64_sync(t_s + 64, h);
+#pragma unroll
+                for (int i = 0; i < 64; ++i) s[64 + i] = h[i];
+            }
             const int first_key = j * kKT;
             if (first_key + kKT - 1 > min_pos) {
 #pragma unroll
@@ -381,13 +407,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
 #pragma unroll
-            for (int i = 4; i < kKT; i += 4) {
-                mx0 = fmaxf(mx0, s[i]);
-                mx1 = fmaxf(mx1, s[i + 1]);
-                mx2 = fmaxf(mx2, s[i + 2]);
-                mx3 = fmaxf(mx3, s[i + 3]);
+            for (int i = 4; i < kKT; i += 8) {
+                mx0 = max3(mx0, s[i], s[i + 4]);
+                mx1 = max3(mx1, s[i + 1], s[i + 5]);
+                mx2 = max3(mx2, s[i + 2], s[i + 6]);
+                mx3 = max3(mx3, s[i + 3], s[i + 7]);
             }
-            const float m_cand = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
+            const float m_cand = max3(fmaxf(mx0, mx1), mx2, mx3) * sl2;
             const bool need = m_cand > m_used + kRescaleThreshold;
             float alpha = 1.f;
             if (need) {
@@ -396,35 +422,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             // a row whose keys in this range are all masked keeps m = -inf and p = 0
             const float neg_m = m_used == -INFINITY ? 0.f : -m_used;
-            float r0 = 0.f, r1 = 0.f, r2 = 0.f, r3 = 0.f;
+            const float2 sl2x2 = make_float2(sl2, sl2), negx2 = make_float2(neg_m, neg_m);
+            float2 ra = make_float2(0.f, 0.f), rb = make_float2(0.f, 0.f);
 #pragma unroll
             for (int i = 0; i < kKT; i += 4) {
-                s[i] = ex2(fmaf(s[i], sl2, neg_m));
-                s[i + 1] = ex2(fmaf(s[i + 1], sl2, neg_m));
-                s[i + 2] = ex2(fmaf(s[i + 2], sl2, neg_m));
-                s[i + 3] = ex2(fmaf(s[i + 3], sl2, neg_m));
-                r0 += s[i];
-                r1 += s[i + 1];
-                r2 += s[i + 2];
-                r3 += s[i + 3];
+                const float2 xa = fma2(make_float2(s[i], s[i + 1]), sl2x2, negx2);
+                const float2 xb = fma2(make_float2(s[i + 2], s[i + 3]), sl2x2, negx2);
+                s[i] = ex2(xa.x);
+                s[i + 1] = ex2(xa.y);
+                s[i + 2] = ex2(xb.x);
+                s[i + 3] = ex2(xb.y);
+                ra = add2(ra, make_float2(s[i], s[i + 1]));
+                rb = add2(rb, make_float2(s[i + 2], s[i + 3]));
             }
-            l_run = l_run * alpha + ((r0 + r1) + (r2 + r3));
-
-            if (jj >= 1) {
-                // P_t(jj-1) consumed and O_t(jj-1) complete
-                ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (jj - 1) & 1, p.err));
-                if (!ok) break;
-                tc_fence_after();
-                if (__any_sync(0xffffffffu, need)) {
+            l_run = l_run * alpha + ((ra.x + ra.y) + (rb.x + rb.y));
+            if (jj >= 1 && __any_sync(0xffffffffu, need)) {
 #pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        float v[32];
-                        tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+                for (int c4 = 0; c4 < 4; ++c4) {
+                    float v[32];
+                    tmem_ld32_sync(t_o + c4 * 32, v);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] *= alpha;
-                        tmem_st32_f(t_lane + kColO + t * 128 + c4 * 32, v);
-                    }
-                    tmem_wait_st();
+                    for (int i = 0; i < 32; ++i) v[i] *= alpha;
+                    tmem_st32_f(t_o + c4 * 32, v);
                 }
             }
             if (j == n_kt_all - 1) {
@@ -435,29 +454,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // zeros again)
                 const int keys_here = min(kKT, sq.ctx_len - first_key);
                 if (keys_here & (kPage - 1)) {
-                    const int s_idx = jj % kNS;
-                    ok = __all_sync(0xffffffffu, mbar_wait(bar(B_VFULL + s_idx), (jj / kNS) & 1, p.err));
+                    const int s_idx = jj % kNV;
+                    ok = __all_sync(0xffffffffu, mbar_wait(bar(B_VFULL + s_idx), (jj / kNV) & 1, p.err));
                     if (!ok) break;
                     const int pg = keys_here / kPage, from = keys_here & (kPage - 1);
                     const int n = (kPage - from) * 8;  // 16-byte chunks per half
-                    uint8_t *vb = sg + kOffV + s_idx * kKVBytes + pg * kBox + from * 128;
+                    uint8_t *vb = sg + kOffV + s_idx * kTileBytes + pg * kBox + from * 128;
                     for (int c = r; c < 2 * n; c += 128)
-                        *reinterpret_cast<uint4 *>(vb + (c / n) * kKVHalf + (c % n) * 16) = make_uint4(0, 0, 0, 0);
+                        *reinterpret_cast<uint4 *>(vb + (c / n) * kHalf + (c % n) * 16) = make_uint4(0, 0, 0, 0);
+                    fence_proxy_async_smem();
                 }
             }
+            // P (bf16 pairs, lower key in the low half) over the first 64 columns of S
 #pragma unroll
-            for (int c = 0; c < kKT / 8; ++c) {
-                uint4 v;
-                v.x = pack_bf16x2(s[8 * c + 0], s[8 * c + 1]);
-                v.y = pack_bf16x2(s[8 * c + 2], s[8 * c + 3]);
-                v.z = pack_bf16x2(s[8 * c + 4], s[8 * c + 5]);
-                v.w = pack_bf16x2(s[8 * c + 6], s[8 * c + 7]);
-                *reinterpret_cast<uint4 *>(prow + ((c ^ (r & 7)) << 4)) = v;
+            for (int h = 0; h < 2; ++h) {
+                uint32_t pk[32];
+#pragma unroll
+                for (int i = 0; i < 32; ++i) pk[i] = pack_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
+                tmem_st32(t_s + 32 * h, pk);
             }
-            fence_proxy_async_smem();
+            tmem_wait_st();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar(B_PFULL + t));
+            if (lane == 0) {
+                mbar_arrive(bar(B_PFULL + t));
+                if (hpc == 2) mbar_arrive(bar(B_TURN + (t ^ 1)));  // the other tile's turn
+            }
         }
 
         if (ok) ok = __all_sync(0xffffffffu, mbar_wait(bar(B_ODONE + t), (n_kt - 1) & 1, p.err));
@@ -470,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int c4 = 0; c4 < 4; ++c4) {
                     float v[32];
-                    tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+                    tmem_ld32_sync(t_o + c4 * 32, v);
                     if (r < rows_valid) store_row32(p, orow, c4, v, inv_l);
                 }
             }
@@ -486,7 +508,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int c4 = 0; c4 < 4; ++c4) {
                     float v[32];
-                    tmem_ld32_sync(t_lane + kColO + t * 128 + c4 * 32, v);
+                    tmem_ld32_sync(t_o + c4 * 32, v);
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
                         __stcg(dst + c4 * 8 + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
@@ -495,7 +517,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __threadfence();
             const int any_fail = named_barrier_or(1, nthr, !ok);
-            int *s_last = reinterpret_cast<int *>(sg + kOffAbort + 4);
+            int *s_last = reinterpret_cast<int *>(sg + kOffLast);
             if (!any_fail) {
                 if (t == 0 && r == 0) {
                     int *ticket = p.tickets + static_cast<int64_t>(wk.part) * slots + slot;
@@ -528,10 +550,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
                             const float mi = __ldcg(p.part_ml + q * 2);
                             const float f = mi == -INFINITY ? 0.f : ex2(mi - M);
-                            const float4 *src = reinterpret_cast<const float4 *>(p.part_o + q * kHeadDim + c4 * 32);
+                            const float4 *srcp = reinterpret_cast<const float4 *>(p.part_o + q * kHeadDim + c4 * 32);
 #pragma unroll
                             for (int c = 0; c < 8; ++c) {
-                                const float4 v = __ldcg(src + c);
+                                const float4 v = __ldcg(srcp + c);
                                 acc[4 * c] += f * v.x;
                                 acc[4 * c + 1] += f * v.y;
                                 acc[4 * c + 2] += f * v.z;
@@ -545,9 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 ok = false;
             }
         }
-        if (!ok) {
-            *abort_flag = 1;
-        }
+        if (!ok) *abort_flag = 1;
       }
     }
 

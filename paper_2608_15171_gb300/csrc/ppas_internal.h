@@ -24,7 +24,7 @@ constexpr int kPageBytes = kPage * kRowBytes;  // one (block, kv-head) page: 4 K
 // Long ranges are split over several CTAs (split-KV); each split writes a
 // partial (m, l, O) and the last CTA of the tile merges them.
 constexpr int kTileQ = 128;            // query tokens per tile (tcgen05 M)
-constexpr int kPrefillKT = 64;         // keys per KV tile
+constexpr int kPrefillKT = 128;        // keys per KV tile
 constexpr int kMaxPrefillSeqs = 128;
 constexpr int kMaxPrefillWork = 1024;  // work items per launch
 // split-KV sizing: a step is cut into about this many CTAs, with at least
