@@ -35,6 +35,31 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// A side stream per device for the decode launch of a mixed step: the
+// prefill kernel goes first on the caller's stream, the decode kernel is
+// forked after it, so decode CTAs fill SMs as prefill CTAs retire.  Events
+// join it back before the call returns.  The mutex serialises the enqueue
+// (the events are shared per device).
+struct SideStream {
+    cudaStream_t stream = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
+};
+std::mutex g_side_mutex;
+SideStream g_side[64];
+
+SideStream *side_stream() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    SideStream &ss = g_side[dev];
+    if (!ss.stream) {
+        if (cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
+        if (cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming) != cudaSuccess)
+            return nullptr;
+    }
+    return &ss;
+}
+
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 }  // namespace
@@ -284,13 +309,13 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         !encode_kv_map(&tm_v, v_cache, num_blocks, n_kv_heads))
         return PPAS_ERR_CUDA;
 
-    // ---------------- decode rows
-    if (!dp.rows.empty()) {
+    auto run_decode = [&](cudaStream_t ds) -> ppas_status {
+        if (dp.rows.empty()) return PPAS_OK;
         uint8_t *ws = static_cast<uint8_t *>(workspace);
         float *part_ml = reinterpret_cast<float *>(ws);
         float *part_o = reinterpret_cast<float *>(ws + dp.ml_bytes);
         int32_t *counters = reinterpret_cast<int32_t *>(ws + dp.ml_bytes + dp.o_bytes);
-        if (cudaMemsetAsync(counters, 0, dp.counter_bytes, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+        if (cudaMemsetAsync(counters, 0, dp.counter_bytes, ds) != cudaSuccess) return PPAS_ERR_CUDA;
         DecodeParams dprm;
         std::memset(&dprm, 0, sizeof(dprm));
         dprm.q = static_cast<const __nv_bfloat16 *>(q);
@@ -326,12 +351,29 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
                 part_base += r.n_splits;
             }
             dprm.n_ctas = cta;
-            if (launch_decode(tm_k, tm_v, dprm, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+            if (launch_decode(tm_k, tm_v, dprm, ds) != cudaSuccess) return PPAS_ERR_CUDA;
         }
-    }
+        return PPAS_OK;
+    };
 
+    // decode rows alone: launch on the caller's stream
+    if (pf.items.empty()) return run_decode(cs);
+
+    // with prefill chunks in the same step the decode launch is forked onto
+    // a side stream after the prefill launch and joined back
+    SideStream *side = dp.rows.empty() ? nullptr : side_stream();
+    std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
+    if (side) {
+        side_lock.lock();
+        if (cudaEventRecord(side->fork, cs) != cudaSuccess ||
+            cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
+            return PPAS_ERR_CUDA;
+    } else if (!dp.rows.empty()) {
+        const ppas_status ds = run_decode(cs);
+        if (ds != PPAS_OK) return ds;
+    }
     // ---------------- prefill chunks
-    if (!pf.items.empty()) {
+    {
         CUtensorMap tm_q;
         if (!encode_q_map(&tm_q, q, static_cast<int32_t>(total_q), n_q_heads)) return PPAS_ERR_CUDA;
         uint8_t *pws = static_cast<uint8_t *>(workspace) + dp.total_bytes();
@@ -379,6 +421,13 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
             w.split = (static_cast<uint32_t>(it.n_splits) << 16) | static_cast<uint32_t>(it.split);
         }
         if (!flush()) return PPAS_ERR_CUDA;
+    }
+    if (side) {
+        const ppas_status ds = run_decode(side->stream);
+        if (ds != PPAS_OK) return ds;
+        if (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
+            cudaStreamWaitEvent(cs, side->join, 0) != cudaSuccess)
+            return PPAS_ERR_CUDA;
     }
     return PPAS_OK;
 }

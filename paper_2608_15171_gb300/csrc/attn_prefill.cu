@@ -500,43 +500,50 @@ __global__ void __launch_bounds__(kThreads, 1)
             // split-KV: write this range's (m, l, O) for the row, then the last
             // CTA of the tile merges every range:
             //   o = sum_i 2^(m_i - M) o_i / sum_i 2^(m_i - M) l_i,  M = max_i m_i
+            // Partial O of one (split, slot, tile) is stored as 4 column chunks
+            // of [128 rows][32 floats], so a warp writes and reads 4 KB
+            // contiguous per chunk.
             const int split = static_cast<int>(wk.split & 0xFFFFu);
-            const int64_t prow = ((static_cast<int64_t>(wk.part + split) * slots + slot) * hpc + t) * kTileQ + r;
+            auto pblk = [&](int i) {  // (split i, slot, tile) block index
+                return (static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t;
+            };
             if (ok) {
                 tc_fence_after();
-                float4 *dst = reinterpret_cast<float4 *>(p.part_o + prow * kHeadDim);
+                const int64_t b = pblk(split);
 #pragma unroll
                 for (int c4 = 0; c4 < 4; ++c4) {
                     float v[32];
                     tmem_ld32_sync(t_o + c4 * 32, v);
+                    float4 *dst = reinterpret_cast<float4 *>(p.part_o + ((b * 4 + c4) * kTileQ + r) * 32);
 #pragma unroll
                     for (int i = 0; i < 8; ++i)
-                        __stcg(dst + c4 * 8 + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
+                        __stcg(dst + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
                 }
-                __stcg(reinterpret_cast<float2 *>(p.part_ml + prow * 2), make_float2(m_used, l_run));
+                __stcg(reinterpret_cast<float2 *>(p.part_ml + (b * kTileQ + r) * 2), make_float2(m_used, l_run));
             }
-            __threadfence();
             const int any_fail = named_barrier_or(1, nthr, !ok);
             int *s_last = reinterpret_cast<int *>(sg + kOffLast);
             if (!any_fail) {
                 if (t == 0 && r == 0) {
+                    // one release at GPU scope covers the warpgroups' writes
+                    // ordered before it by the barrier (fences are cumulative)
+                    __threadfence();
                     int *ticket = p.tickets + static_cast<int64_t>(wk.part) * slots + slot;
                     const int prev = atomicAdd(ticket, 1);
-                    *s_last = (prev == n_splits - 1);
-                    if (prev == n_splits - 1) *ticket = 0;  // ready for the next call
+                    const int last = prev == n_splits - 1;
+                    if (last) {
+                        *ticket = 0;  // ready for the next call
+                        __threadfence();
+                    }
+                    *reinterpret_cast<volatile int *>(s_last) = last;
                 }
                 named_barrier_sync(1, nthr);
                 if (*reinterpret_cast<volatile int *>(s_last)) {
-                    __threadfence();
                     float M = -INFINITY;
-                    for (int i = 0; i < n_splits; ++i) {
-                        const int64_t q = ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
-                        M = fmaxf(M, __ldcg(p.part_ml + q * 2));
-                    }
+                    for (int i = 0; i < n_splits; ++i) M = fmaxf(M, __ldcg(p.part_ml + (pblk(i) * kTileQ + r) * 2));
                     float L = 0.f;
                     for (int i = 0; i < n_splits; ++i) {
-                        const int64_t q = ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
-                        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + q * 2));
+                        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + (pblk(i) * kTileQ + r) * 2));
                         L += (ml.x == -INFINITY ? 0.f : ex2(ml.x - M)) * ml.y;
                     }
                     const float inv_l = 1.f / L;
@@ -545,19 +552,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                         float acc[32];
 #pragma unroll
                         for (int c = 0; c < 32; ++c) acc[c] = 0.f;
-                        for (int i = 0; i < n_splits; ++i) {
-                            const int64_t q =
-                                ((static_cast<int64_t>(wk.part + i) * slots + slot) * hpc + t) * kTileQ + r;
-                            const float mi = __ldcg(p.part_ml + q * 2);
-                            const float f = mi == -INFINITY ? 0.f : ex2(mi - M);
-                            const float4 *srcp = reinterpret_cast<const float4 *>(p.part_o + q * kHeadDim + c4 * 32);
+                        // two splits per round: 16 independent 16-byte loads in flight
+                        for (int i = 0; i < n_splits; i += 2) {
+                            const int i1 = min(i + 1, n_splits - 1);
+                            const float m0 = __ldcg(p.part_ml + (pblk(i) * kTileQ + r) * 2);
+                            const float m1 = __ldcg(p.part_ml + (pblk(i1) * kTileQ + r) * 2);
+                            const float f0 = m0 == -INFINITY ? 0.f : ex2(m0 - M);
+                            const float f1 = (i1 == i || m1 == -INFINITY) ? 0.f : ex2(m1 - M);
+                            const float4 *a0 = reinterpret_cast<const float4 *>(p.part_o + ((pblk(i) * 4 + c4) * kTileQ + r) * 32);
+                            const float4 *a1 = reinterpret_cast<const float4 *>(p.part_o + ((pblk(i1) * 4 + c4) * kTileQ + r) * 32);
+                            float4 v0[8], v1[8];
 #pragma unroll
                             for (int c = 0; c < 8; ++c) {
-                                const float4 v = __ldcg(srcp + c);
-                                acc[4 * c] += f * v.x;
-                                acc[4 * c + 1] += f * v.y;
-                                acc[4 * c + 2] += f * v.z;
-                                acc[4 * c + 3] += f * v.w;
+                                v0[c] = __ldcg(a0 + c);
+                                v1[c] = __ldcg(a1 + c);
+                            }
+#pragma unroll
+                            for (int c = 0; c < 8; ++c) {
+                                acc[4 * c] += f0 * v0[c].x + f1 * v1[c].x;
+                                acc[4 * c + 1] += f0 * v0[c].y + f1 * v1[c].y;
+                                acc[4 * c + 2] += f0 * v0[c].z + f1 * v1[c].z;
+                                acc[4 * c + 3] += f0 * v0[c].w + f1 * v1[c].w;
                             }
                         }
                         if (r < rows_valid) store_row32(p, orow, c4, acc, inv_l);

@@ -59,7 +59,7 @@ struct PrefillParams {
     int32_t heads_per_cta;  // 2 when the group has >= 2 heads, else 1
     float scale_log2;       // scale * log2(e)
     int32_t *err;
-    float *part_o;          // [n_part, slots, heads_per_cta, 128 rows, 128]
+    float *part_o;          // [n_part, slots, heads_per_cta, 4 chunks, 128 rows, 32]
     float *part_ml;         // [n_part, slots, heads_per_cta, 128 rows, 2]
     int32_t *tickets;       // [n_part, slots] (first slot of each split tile)
     int32_t n_work;         // work items in this launch; grid = n_work * slots
