@@ -230,6 +230,13 @@ ppas_status ppas_attention_step_noalloc(const void *q, const void *k_cache, cons
                                         int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
                                         int32_t out_is_fp32, int32_t *d_err_flag, void *stream);
 
+/* Failure-path check (device).  Launches one thread that waits, with a
+ * limit of limit_us microseconds (1 .. 2,000,000), on a barrier nothing
+ * arrives on -- the same bounded wait every kernel of this library uses --
+ * so that the wait runs out and PPAS_DEVERR_TIMEOUT is written to
+ * *d_err_flag (device int32, required).  The GPU context stays usable. */
+ppas_status ppas_debug_wait_timeout(int32_t *d_err_flag, uint32_t limit_us, void *stream);
+
 /* Static description of a status code (never NULL). */
 const char *ppas_status_string(ppas_status status);
 

@@ -243,6 +243,14 @@ extern "C" const char *ppas_status_string(ppas_status s) {
 
 extern "C" int32_t ppas_abi_version(void) { return 1; }
 
+extern "C" ppas_status ppas_debug_wait_timeout(int32_t *d_err_flag, uint32_t limit_us, void *stream) {
+    if (!d_err_flag || limit_us < 1 || limit_us > 2000000) return PPAS_ERR_INVALID_ARG;
+    return launch_wait_timeout(d_err_flag, static_cast<unsigned long long>(limit_us) * 1000ull,
+                               static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? PPAS_OK
+               : PPAS_ERR_CUDA;
+}
+
 extern "C" ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *d_slot_mapping,
                                       int32_t n_tokens, void *k_cache, void *v_cache, int32_t num_blocks,
                                       int32_t n_kv_heads, int32_t head_dim, int32_t *d_err_flag, void *stream) {

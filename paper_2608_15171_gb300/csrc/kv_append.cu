@@ -36,6 +36,22 @@ __global__ void __launch_bounds__(256) kv_append_kernel(const uint4 *__restrict_
     }
 }
 
+// One thread waits on an mbarrier that nothing arrives on; the bounded wait
+// gives up after limit_ns and records PPAS_DEVERR_TIMEOUT.  Exercises the
+// failure path every kernel wait shares, without faulting or hanging.
+__global__ void wait_timeout_kernel(int32_t *err, unsigned long long limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    const uint32_t b = smem_u32(&bar);
+    mbar_init(b, 1);
+    fence_mbar_init();
+    mbar_wait(b, 0, err, limit_ns);
+}
+
+cudaError_t launch_wait_timeout(int32_t *err, unsigned long long limit_ns, cudaStream_t st) {
+    wait_timeout_kernel<<<1, 1, 0, st>>>(err, limit_ns);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_kv_append(const void *k_new, const void *v_new, const int32_t *slots, int32_t n_tokens,
                              void *k_cache, void *v_cache, int32_t num_blocks, int32_t n_kv_heads,
                              int32_t head_dim, int32_t *err, cudaStream_t st) {

@@ -142,6 +142,8 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
 int32_t device_sm_count();
 
 // launchers (return a cudaError_t of the launch)
+cudaError_t launch_wait_timeout(int32_t *err, unsigned long long limit_ns, cudaStream_t st);
+
 cudaError_t launch_kv_append(const void *k_new, const void *v_new, const int32_t *slots, int32_t n_tokens,
                              void *k_cache, void *v_cache, int32_t num_blocks, int32_t n_kv_heads,
                              int32_t head_dim, int32_t *err, cudaStream_t st);

@@ -35,7 +35,8 @@ PPAS_REQ_PENDING, PPAS_REQ_WAITING, PPAS_REQ_RUNNING, PPAS_REQ_FINISHED = 0, 1, 
 
 EXPORTED = ("ppas_sched_create", "ppas_sched_destroy", "ppas_sched_free_blocks", "ppas_plan_step",
             "ppas_kv_append", "ppas_attention_workspace_size", "ppas_attention_step",
-            "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc")
+            "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc",
+            "ppas_debug_wait_timeout")
 PPAS_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
 
 
@@ -85,6 +86,8 @@ _lib.ppas_attention_step_noalloc.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void
                                              _c.c_int32, _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p,
                                              _c.c_void_p]
 _lib.ppas_attention_step_noalloc.restype = _c.c_int32
+_lib.ppas_debug_wait_timeout.argtypes = [_c.c_void_p, _c.c_uint32, _c.c_void_p]
+_lib.ppas_debug_wait_timeout.restype = _c.c_int32
 _lib.ppas_status_string.argtypes = [_c.c_int32]
 _lib.ppas_status_string.restype = _c.c_char_p
 _lib.ppas_abi_version.argtypes = []
@@ -196,6 +199,10 @@ def ppas_attention_step_noalloc(q, k_cache, v_cache, num_blocks: int, d_block_ta
                                             float(scale), _ptr(out), 1 if out_is_fp32 else 0, _ptr(d_err_flag),
                                             _stream(stream)),
            "ppas_attention_step_noalloc")
+
+
+def ppas_debug_wait_timeout(d_err_flag, limit_us: int, stream=None) -> None:
+    _check(_lib.ppas_debug_wait_timeout(_ptr(d_err_flag), int(limit_us), _stream(stream)), "ppas_debug_wait_timeout")
 
 
 # ---------------------------------------------------------------- planner object
