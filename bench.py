@@ -249,6 +249,17 @@ def _roofline_time_us(shape, geo, peaks, sustained=True):
     return max(wl.step_flops(shape, geo) / tf, wl.step_bytes(shape, geo) / bw) * 1e6
 
 
+def _max_over_ranks(dist, x):
+    """The largest x over all ranks, on every rank (x itself without a process group)."""
+    if dist is None:
+        return x
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def _timed(torch, dist, fn, steps, warmup, stream, rank, sample_clocks):
     for _ in range(warmup):
         fn(None)
@@ -273,9 +284,7 @@ def _timed(torch, dist, fn, steps, warmup, stream, rank, sample_clocks):
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+        ms = _max_over_ranks(dist, ms)
         dist.barrier()
     clocks = sampler.stop() if sampler else None
     return ms, timers, launches, clocks
