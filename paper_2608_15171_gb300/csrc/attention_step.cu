@@ -15,9 +15,19 @@ namespace ppas {
 namespace {
 
 // Decode rows are split so that one step launches about this many CTAs
-// (one per SM on a 152-SM GB300).  A fixed number keeps the workspace size a
-// pure function of the step's lengths.
-constexpr int64_t kDecodeTargetCtas = 152;
+// (one per SM).
+constexpr int64_t kDecodeTargetCtas = kPlanSms;
+
+// Throughput model behind the SMs the prefill kernel leaves to the decode
+// launch (measured on GB300): one item's KV tile (two q-heads x 128 queries x
+// 128 keys) takes about 2.06 us of one SM; next to a running prefill kernel
+// the decode kernel streams 65-80 GB/s per SM (the upper figure is used, so
+// that a wrong estimate leaves decode rows rather than prefill items as the
+// tail: the slower side of the balance), and at most kDecodeBytesPerUs on
+// the GPU.
+constexpr double kPrefillTileUs = 2.06;
+constexpr double kDecodeBytesPerSmUs = 8.0e4;
+constexpr double kDecodeBytesPerUs = 4.35e6;
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -139,49 +149,160 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
 }
 
 PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                         int32_t n_kv_heads, bool allow_split) {
+                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas) {
     PrefillPlan pf;
     const int32_t g = n_q_heads / n_kv_heads;
     pf.heads_per_cta = g >= 2 ? 2 : 1;
     pf.slots = n_q_heads / pf.heads_per_cta;
-    struct Tile {
-        int32_t seq, qt, n_kt;
+    n_ctas = std::max(1, std::min(n_ctas, kMaxPrefillCtas));
+    struct Unit {
+        int32_t seq, qt, slot, n_kt;
     };
-    std::vector<Tile> tiles;
-    int64_t total = 0;
+    std::vector<Unit> units;
     for (int32_t s = 0; s < n_seqs; ++s) {
         if (q_lens[s] == 1) continue;
         const int32_t prefix = ctx_lens[s] - q_lens[s];
         const int32_t n_qt = (q_lens[s] + kTileQ - 1) / kTileQ;
         for (int32_t t = 0; t < n_qt; ++t) {
             const int32_t last = prefix + std::min(q_lens[s], (t + 1) * kTileQ) - 1;
-            tiles.push_back({s, t, last / kPrefillKT + 1});
-            total += static_cast<int64_t>(last / kPrefillKT + 1) * pf.slots;
+            for (int32_t sl = 0; sl < pf.slots; ++sl) units.push_back({s, t, sl, last / kPrefillKT + 1});
         }
     }
-    int64_t per_cta = (total + kPrefillTargetCtas - 1) / kPrefillTargetCtas;
-    per_cta = std::max<int64_t>(per_cta, kPrefillMinSplitTiles);
-    for (const Tile &t : tiles) {
-        int32_t ns = 1;
-        if (allow_split)
-            ns = static_cast<int32_t>(std::min<int64_t>(kPrefillMaxSplits, (t.n_kt + per_cta - 1) / per_cta));
-        const int32_t part = ns > 1 ? static_cast<int32_t>(pf.n_part) : -1;
-        for (int32_t i = 0; i < ns; ++i) {
-            const int32_t kt0 = static_cast<int32_t>(static_cast<int64_t>(t.n_kt) * i / ns);
-            const int32_t kt1 = static_cast<int32_t>(static_cast<int64_t>(t.n_kt) * (i + 1) / ns);
-            pf.items.push_back({t.seq, t.qt, kt0, kt1, part, i, ns});
+    if (units.empty()) return pf;
+    // longest first
+    std::stable_sort(units.begin(), units.end(), [](const Unit &a, const Unit &b) { return a.n_kt > b.n_kt; });
+
+    size_t u0 = 0;
+    while (u0 < units.size()) {
+        // a launch takes consecutive units while its tables have room (every
+        // CTA boundary adds at most one item)
+        PrefillLaunchPlan lp;
+        std::vector<int32_t> local(n_seqs, -1);
+        size_t u1 = u0;
+        for (; u1 < units.size(); ++u1) {
+            const bool new_seq = local[units[u1].seq] < 0;
+            if (u1 - u0 + static_cast<size_t>(n_ctas) > static_cast<size_t>(kMaxPrefillWork)) break;
+            if (new_seq && lp.seqs.size() == static_cast<size_t>(kMaxPrefillSeqs)) break;
+            if (new_seq) {
+                local[units[u1].seq] = static_cast<int32_t>(lp.seqs.size());
+                lp.seqs.push_back(units[u1].seq);
+            }
         }
-        if (ns > 1) pf.n_part += ns;
+        int64_t total = 0, tiles = 0;
+        for (size_t u = u0; u < u1; ++u) {
+            total += units[u].n_kt + kPrefillItemCost;
+            tiles += units[u].n_kt;
+        }
+        auto item = [&](const Unit &u, int32_t kt0, int32_t kt1) {
+            return PrefillWork{static_cast<uint16_t>(u.qt), static_cast<uint8_t>(local[u.seq]),
+                               static_cast<uint8_t>(u.slot), static_cast<uint16_t>(kt0), static_cast<uint16_t>(kt1),
+                               kNoPart, 0};
+        };
+        // whole units, longest first, each to the least loaded CTA
+        const int32_t nc_whole = static_cast<int32_t>(std::min<int64_t>(n_ctas, u1 - u0));
+        std::vector<std::vector<PrefillWork>> whole(nc_whole);
+        int64_t whole_span = 0;
+        {
+            std::vector<std::pair<int64_t, int32_t>> heap;  // (load, cta), min-heap
+            for (int32_t c = 0; c < nc_whole; ++c) heap.push_back({0, c});
+            auto later = [](const std::pair<int64_t, int32_t> &a, const std::pair<int64_t, int32_t> &b) {
+                return a.first != b.first ? a.first > b.first : a.second > b.second;
+            };
+            std::make_heap(heap.begin(), heap.end(), later);
+            for (size_t u = u0; u < u1; ++u) {
+                std::pop_heap(heap.begin(), heap.end(), later);
+                auto &top = heap.back();
+                whole[top.second].push_back(item(units[u], 0, units[u].n_kt));
+                top.first += units[u].n_kt + kPrefillItemCost;
+                whole_span = std::max(whole_span, top.first);
+                std::push_heap(heap.begin(), heap.end(), later);
+            }
+        }
+        // cutting units evens the CTAs out at the cost of partials and a
+        // merge; it is taken when it shortens the launch by more than that
+        const int32_t nc = static_cast<int32_t>(std::min<int64_t>(n_ctas, tiles));
+        const int64_t cut_span = (total + static_cast<int64_t>(nc - 1) * kPrefillItemCost + nc - 1) / nc;
+        const bool cut = allow_split && cut_span + kPrefillMergeCost < whole_span;
+        std::vector<std::vector<PrefillWork>> per_cta;
+        if (cut) {
+            per_cta.resize(nc);
+            // stream-K: CTA c gets the cost range [total c / nc, total (c + 1) / nc)
+            // of the units laid end to end; a unit is cut where a range ends,
+            // and every cut adds one item's cost
+            total += static_cast<int64_t>(nc - 1) * kPrefillItemCost;
+            int32_t cta = 0;
+            int64_t pos = 0;  // cost handed out so far
+            for (size_t u = u0; u < u1; ++u) {
+                const Unit &un = units[u];
+                std::vector<std::pair<int32_t, PrefillWork>> pieces;  // (cta, item)
+                int32_t a = 0;
+                while (a < un.n_kt) {
+                    const int64_t end = total * (cta + 1) / nc;
+                    const int64_t room = end - pos - kPrefillItemCost;
+                    const int32_t left = un.n_kt - a;
+                    int32_t take = left;
+                    if (cta < nc - 1 && room < left) {
+                        if (room < kPrefillMinPiece) {  // too little left in this CTA's range
+                            ++cta;
+                            continue;
+                        }
+                        take = static_cast<int32_t>(room);
+                        if (left - take < kPrefillMinPiece) take = left;  // no sliver for the next CTA
+                    }
+                    pieces.push_back({cta, item(un, a, a + take)});
+                    pos += take + kPrefillItemCost;
+                    a += take;
+                }
+                if (pieces.size() > 1) {
+                    lp.split_units.push_back({un.seq, un.qt, un.slot, static_cast<int32_t>(pieces.size()), lp.n_part});
+                    for (auto &pc : pieces) pc.second.part = static_cast<uint16_t>(lp.n_part++);
+                }
+                for (auto &pc : pieces) per_cta[pc.first].push_back(pc.second);
+            }
+        } else {
+            per_cta = std::move(whole);
+        }
+        lp.cta_begin.push_back(0);
+        for (size_t c = 0; c < per_cta.size(); ++c) {
+            if (per_cta[c].empty()) continue;  // (a CTA with nothing is left out)
+            lp.work.insert(lp.work.end(), per_cta[c].begin(), per_cta[c].end());
+            lp.cta_begin.push_back(static_cast<uint16_t>(lp.work.size()));
+        }
+        pf.n_part = std::max<int64_t>(pf.n_part, lp.n_part);
+        pf.launches.push_back(std::move(lp));
+        u0 = u1;
     }
-    // heaviest first: the block scheduler hands them out first
-    std::stable_sort(pf.items.begin(), pf.items.end(), [](const PrefillItem &a, const PrefillItem &b) {
-        return (a.kt1 - a.kt0) > (b.kt1 - b.kt0);
-    });
-    const size_t per_part = static_cast<size_t>(pf.slots) * pf.heads_per_cta * kTileQ;
+    const size_t per_part = static_cast<size_t>(pf.heads_per_cta) * kTileQ;
     pf.o_bytes = align256(static_cast<size_t>(pf.n_part) * per_part * kHeadDim * sizeof(float));
     pf.ml_bytes = align256(static_cast<size_t>(pf.n_part) * per_part * 2 * sizeof(float));
-    pf.ticket_bytes = align256(static_cast<size_t>(pf.n_part) * pf.slots * sizeof(int32_t));
     return pf;
+}
+
+int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                           int32_t n_kv_heads) {
+    const int32_t hpc = n_q_heads / n_kv_heads >= 2 ? 2 : 1;
+    const int64_t slots = n_q_heads / hpc;
+    double units = 0.0, bytes = 0.0;  // prefill KV tiles x head slots, decode K/V bytes
+    for (int32_t s = 0; s < n_seqs; ++s) {
+        if (q_lens[s] == 1) {
+            bytes += static_cast<double>((ctx_lens[s] + kPage - 1) / kPage) * kPageBytes * 2 * n_kv_heads;
+            continue;
+        }
+        const int32_t prefix = ctx_lens[s] - q_lens[s];
+        const int32_t n_qt = (q_lens[s] + kTileQ - 1) / kTileQ;
+        for (int32_t t = 0; t < n_qt; ++t) {
+            const int32_t last = prefix + std::min(q_lens[s], (t + 1) * kTileQ) - 1;
+            units += static_cast<double>(last / kPrefillKT + 1) * slots;
+        }
+    }
+    if (units == 0.0 || bytes == 0.0) return 0;
+    // the decode launch streams on k SMs while the prefill kernel runs on
+    // the rest; the smallest k that finishes the decode rows by the time the
+    // prefill items are done:  k r T(k) >= bytes,  T(k) = units tau / (S - k)
+    const double sm_time = units * kPrefillTileUs;
+    int32_t k = static_cast<int32_t>(std::ceil(bytes * kPlanSms / (kDecodeBytesPerSmUs * sm_time + bytes)));
+    k = std::min(k, static_cast<int32_t>(kDecodeBytesPerUs / kDecodeBytesPerSmUs));
+    return std::max(0, std::min(k, kPlanSms / 2));
 }
 
 size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
@@ -209,9 +330,12 @@ ppas_status check_step(const void *q, const void *k_cache, const void *v_cache, 
     if (n_q_heads % n_kv_heads != 0) return PPAS_ERR_INVALID_ARG;
     const int32_t g = n_q_heads / n_kv_heads;
     if (g != 1 && g != 2 && g != 4 && g != 8) return PPAS_ERR_UNSUPPORTED;
+    if (n_q_heads / (g >= 2 ? 2 : 1) > 256) return PPAS_ERR_UNSUPPORTED;  // head slots of the prefill items
     int64_t tq = 0;
     for (int32_t s = 0; s < n_seqs; ++s) {
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return PPAS_ERR_INVALID_ARG;
+        // KV tile indices of the prefill items are 16-bit
+        if (h_q_lens[s] > 1 && h_ctx_lens[s] > 65535 * kPrefillKT) return PPAS_ERR_UNSUPPORTED;
         if (static_cast<int64_t>(h_ctx_lens[s]) > static_cast<int64_t>(max_blocks_per_seq) * kPage)
             return PPAS_ERR_INVALID_ARG;
         tq += h_q_lens[s];
@@ -271,8 +395,9 @@ extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h
         return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return 0;
+    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
     return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes() +
-           plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true).total_bytes();
+           plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas).total_bytes();
 }
 
 extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
@@ -302,10 +427,11 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     }
 
     DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
-    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true);
+    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
+    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
     // a workspace too small for the prefill splits runs the prefill tiles unsplit
     if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
-        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false);
+        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false, n_ctas);
     const size_t need = dp.total_bytes() + pf.total_bytes();
     if (need > 0) {
         if (!workspace || workspace_bytes < need) return PPAS_ERR_CAPACITY;
@@ -365,7 +491,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     };
 
     // decode rows alone: launch on the caller's stream
-    if (pf.items.empty()) return run_decode(cs);
+    if (pf.empty()) return run_decode(cs);
 
     // with prefill chunks in the same step the decode launch is forked onto
     // a side stream after the prefill launch and joined back
@@ -401,34 +527,40 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         if (pf.n_part > 0) {
             pp.part_o = reinterpret_cast<float *>(pws);
             pp.part_ml = reinterpret_cast<float *>(pws + pf.o_bytes);
-            pp.tickets = reinterpret_cast<int32_t *>(pws + pf.o_bytes + pf.ml_bytes);
-            if (cudaMemsetAsync(pp.tickets, 0, pf.ticket_bytes, cs) != cudaSuccess) return PPAS_ERR_CUDA;
         }
-        std::vector<int32_t> local(n_seqs, -1);
-        int32_t n_local = 0;
-        auto flush = [&]() -> bool {
-            if (pp.n_work == 0) return true;
-            const bool ok = launch_prefill(tm_q, tm_k, tm_v, pp, cs) == cudaSuccess;
-            pp.n_work = 0;
-            std::fill(local.begin(), local.end(), -1);
-            n_local = 0;
-            return ok;
-        };
-        for (const PrefillItem &it : pf.items) {
-            if (pp.n_work == kMaxPrefillWork || (local[it.seq] < 0 && n_local == kMaxPrefillSeqs))
-                if (!flush()) return PPAS_ERR_CUDA;
-            if (local[it.seq] < 0) {
-                local[it.seq] = n_local;
-                pp.seqs[n_local] = {q_start[it.seq], h_q_lens[it.seq], h_ctx_lens[it.seq], it.seq};
-                ++n_local;
+        MergeParams mp;
+        std::memset(&mp, 0, sizeof(mp));
+        mp.part_o = pp.part_o;
+        mp.part_ml = pp.part_ml;
+        mp.out = out;
+        mp.out_fp32 = pp.out_fp32;
+        mp.n_q_heads = n_q_heads;
+        mp.heads_per_cta = pf.heads_per_cta;
+        for (const PrefillLaunchPlan &lp : pf.launches) {
+            for (size_t i = 0; i < lp.seqs.size(); ++i) {
+                const int32_t sq = lp.seqs[i];
+                pp.seqs[i] = {q_start[sq], h_q_lens[sq], h_ctx_lens[sq], sq};
             }
-            PrefillWork &w = pp.work[pp.n_work++];
-            w.seq_qt = (static_cast<uint32_t>(local[it.seq]) << 16) | static_cast<uint32_t>(it.qt);
-            w.kt_range = (static_cast<uint32_t>(it.kt0) << 16) | static_cast<uint32_t>(it.kt1);
-            w.part = it.part;
-            w.split = (static_cast<uint32_t>(it.n_splits) << 16) | static_cast<uint32_t>(it.split);
+            std::memcpy(pp.work, lp.work.data(), lp.work.size() * sizeof(PrefillWork));
+            std::memcpy(pp.cta_begin, lp.cta_begin.data(), lp.cta_begin.size() * sizeof(uint16_t));
+            pp.n_ctas = static_cast<int32_t>(lp.cta_begin.size()) - 1;
+            if (launch_prefill(tm_q, tm_k, tm_v, pp, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+            // the split units' partials are merged once the launch is done
+            for (size_t i0 = 0; i0 < lp.split_units.size(); i0 += kMaxMergeUnits) {
+                const size_t i1 = std::min(lp.split_units.size(), i0 + kMaxMergeUnits);
+                mp.n_units = static_cast<int32_t>(i1 - i0);
+                for (size_t i = i0; i < i1; ++i) {
+                    const PrefillSplitUnit &su = lp.split_units[i];
+                    MergeUnit &mu = mp.units[i - i0];
+                    mu.out_row0 = q_start[su.seq] + su.qt * kTileQ;
+                    mu.part = su.part;
+                    mu.rows_valid = static_cast<uint16_t>(std::min(kTileQ, h_q_lens[su.seq] - su.qt * kTileQ));
+                    mu.n_splits = static_cast<uint16_t>(su.n_splits);
+                    mu.head0 = static_cast<uint16_t>(su.slot * pf.heads_per_cta);
+                }
+                if (launch_prefill_merge(mp, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+            }
         }
-        if (!flush()) return PPAS_ERR_CUDA;
     }
     if (side) {
         const ppas_status ds = run_decode(side->stream);

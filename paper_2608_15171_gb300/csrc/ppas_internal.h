@@ -17,21 +17,28 @@ constexpr int kPage = PPAS_PAGE_TOKENS;        // tokens per KV block
 constexpr int kHeadDim = 128;                  // the only head size with kernels
 constexpr int kRowBytes = kHeadDim * 2;        // one bf16 K or V row
 constexpr int kPageBytes = kPage * kRowBytes;  // one (block, kv-head) page: 4 KB
+// SMs the step plans are made for (GB300).  A fixed number keeps every plan,
+// and so the workspace size, a pure function of the step's lengths.
+constexpr int32_t kPlanSms = 152;
 
 // ------------------------------------------------------------------ prefill
-// Rows with q_len > 1.  One CTA computes one 128-token query tile of
-// heads_per_cta q-heads of one kv-head over a range of its causal KV tiles.
-// Long ranges are split over several CTAs (split-KV); each split writes a
-// partial (m, l, O) and the last CTA of the tile merges them.
-constexpr int kTileQ = 128;            // query tokens per tile (tcgen05 M)
-constexpr int kPrefillKT = 128;        // keys per KV tile
-constexpr int kMaxPrefillSeqs = 128;
-constexpr int kMaxPrefillWork = 1024;  // work items per launch
-// split-KV sizing: a step is cut into about this many CTAs, with at least
-// kPrefillMinSplitTiles KV tiles per CTA and at most kPrefillMaxSplits per tile
-constexpr int64_t kPrefillTargetCtas = 304;
-constexpr int kPrefillMinSplitTiles = 16;
-constexpr int kPrefillMaxSplits = 64;
+// Rows with q_len > 1.  The kernel is persistent: one CTA per SM works
+// through a list of items, each one 128-token query tile of heads_per_cta
+// q-heads of one kv-head (a "head slot") over a range of its causal KV
+// tiles.  The host lays the (tile, head slot) units end to end, longest
+// first, and cuts the line into one equal segment per CTA (stream-K style),
+// so a unit is split only where a segment ends.  Each piece of a split unit
+// writes a partial (m, l, O) and a merge kernel launched after the prefill
+// kernel combines them.
+constexpr int kTileQ = 128;             // query tokens per tile (tcgen05 M)
+constexpr int kPrefillKT = 128;         // keys per KV tile
+constexpr int kMaxPrefillSeqs = 128;    // per launch
+constexpr int kMaxPrefillWork = 2400;   // items per launch (bounded by the 32 KB parameter space)
+constexpr int kMaxPrefillCtas = 256;    // CTAs per launch (one per SM)
+constexpr int kPrefillItemCost = 3;     // per-item overhead (Q load, pipeline fill, epilogue), in KV tiles
+constexpr int kPrefillMinPiece = 4;     // shortest piece of a split unit, in KV tiles
+constexpr int kPrefillMergeCost = 4;    // partial writes and the merge launch, in KV tiles
+constexpr uint16_t kNoPart = 0xFFFF;    // an item of an unsplit unit
 
 struct PrefillSeq {
     int32_t q_start;   // first row of the sequence in packed q / out
@@ -40,12 +47,15 @@ struct PrefillSeq {
     int32_t table_row; // row of d_block_tables
 };
 
-struct PrefillWork {
-    uint32_t seq_qt;    // (launch-local sequence << 16) | q tile
-    uint32_t kt_range;  // (first KV tile << 16) | end KV tile (exclusive)
-    int32_t part;       // first partial slot of this tile's splits; -1: not split
-    uint32_t split;     // (number of splits << 16) | this split
+struct PrefillWork {     // one item: (sequence, q tile, head slot, KV range)
+    uint16_t qt;         // q tile within the sequence
+    uint8_t seq;         // launch-local sequence
+    uint8_t slot;        // q-heads slot * heads_per_cta ... + heads_per_cta - 1
+    uint16_t kt0, kt1;   // KV tiles [kt0, kt1)
+    uint16_t part;       // partial slot (launch-relative); kNoPart: unsplit
+    uint16_t pad;
 };
+static_assert(sizeof(PrefillWork) == 12, "compact work item");
 
 struct PrefillParams {
     const int32_t *block_tables;
@@ -59,28 +69,70 @@ struct PrefillParams {
     int32_t heads_per_cta;  // 2 when the group has >= 2 heads, else 1
     float scale_log2;       // scale * log2(e)
     int32_t *err;
-    float *part_o;          // [n_part, slots, heads_per_cta, 4 chunks, 128 rows, 32]
-    float *part_ml;         // [n_part, slots, heads_per_cta, 128 rows, 2]
-    int32_t *tickets;       // [n_part, slots] (first slot of each split tile)
-    int32_t n_work;         // work items in this launch; grid = n_work * slots
-    PrefillWork work[kMaxPrefillWork];  // heaviest first
+    float *part_o;          // [n_part, heads_per_cta, 4 chunks, 128 rows, 32]
+    float *part_ml;         // [n_part, heads_per_cta, 128 rows, 2]
+    int32_t n_ctas;         // grid size
+    uint16_t cta_begin[kMaxPrefillCtas + 1];  // CTA c runs work[cta_begin[c] .. cta_begin[c + 1])
+    PrefillWork work[kMaxPrefillWork];
     PrefillSeq seqs[kMaxPrefillSeqs];
 };
+static_assert(sizeof(PrefillParams) + 3 * 128 <= 32764, "kernel parameter space");
 
-struct PrefillItem {
-    int32_t seq, qt, kt0, kt1, part, split, n_splits;
+// Merge of the split units' partials, launched after the prefill kernel:
+// one thread per (split unit, head of the slot, query row, 4 columns).
+constexpr int kMaxMergeUnits = 1024;  // split units per merge launch
+
+struct MergeUnit {
+    int32_t out_row0;     // packed row of the tile's first query token
+    int32_t part;         // first partial slot of the unit's pieces
+    uint16_t rows_valid;  // query tokens of the tile
+    uint16_t n_splits;    // pieces
+    uint16_t head0;       // first q-head of the slot
+    uint16_t pad;
+};
+
+struct MergeParams {
+    const float *part_o;  // layouts as in PrefillParams
+    const float *part_ml;
+    void *out;
+    int32_t out_fp32;
+    int32_t n_q_heads;
+    int32_t heads_per_cta;
+    int32_t n_units;
+    MergeUnit units[kMaxMergeUnits];
+};
+
+struct PrefillSplitUnit {
+    int32_t seq, qt, slot, n_splits, part;
+};
+
+// one launch of the prefill kernel, as planned on the host
+struct PrefillLaunchPlan {
+    std::vector<int32_t> seqs;          // global sequence index per launch-local sequence
+    std::vector<PrefillWork> work;      // grouped by CTA, in each CTA's order
+    std::vector<uint16_t> cta_begin;    // n_ctas + 1 entries
+    std::vector<PrefillSplitUnit> split_units;  // units of this launch cut into several pieces
+    int32_t n_part = 0;                 // partial slots of this launch
 };
 
 struct PrefillPlan {
-    std::vector<PrefillItem> items;  // sorted heaviest first
-    int64_t n_part = 0;
+    std::vector<PrefillLaunchPlan> launches;
+    int64_t n_part = 0;                 // most partial slots of one launch (the merge follows each launch)
     int32_t slots = 0, heads_per_cta = 1;
-    size_t o_bytes = 0, ml_bytes = 0, ticket_bytes = 0;
-    size_t total_bytes() const { return o_bytes + ml_bytes + ticket_bytes; }
+    size_t o_bytes = 0, ml_bytes = 0;
+    bool empty() const { return launches.empty(); }
+    size_t total_bytes() const { return o_bytes + ml_bytes; }
 };
 
+// SMs the persistent prefill kernel leaves to the decode launch of the same
+// step (0 without decode rows or without prefill chunks)
+int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                           int32_t n_kv_heads);
+
+// n_ctas: CTAs (SMs) the persistent kernel may occupy; allow_split == false
+// keeps every unit whole (no workspace)
 PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                         int32_t n_kv_heads, bool allow_split);
+                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas);
 
 // ------------------------------------------------------------------ decode
 // Rows with q_len == 1.  One CTA handles one (row, kv-head, split): the
@@ -148,6 +200,7 @@ cudaError_t launch_kv_append(const void *k_new, const void *v_new, const int32_t
                              void *k_cache, void *v_cache, int32_t num_blocks, int32_t n_kv_heads,
                              int32_t head_dim, int32_t *err, cudaStream_t st);
 
+cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st);
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
                            const PrefillParams &p, cudaStream_t st);
 
