@@ -135,6 +135,9 @@ def _setup_low(torch, ppas, geo, dev, seed=0):
         W.vn.append([wl.bf16_normal((sh.total_q, hk, D), s + 21 + i, dev) for i, sh in enumerate(shapes)])
         W.out.append([torch.empty((sh.total_q, hq, D), dtype=torch.bfloat16, device=dev) for sh in shapes])
     W.err = torch.zeros(1, dtype=torch.int32, device=dev)
+    # one workspace, sized for the larger of the two iterations
+    W.ws_bytes = max(ppas.ppas_attention_workspace_size(sh.q_lens, sh.ctx_lens, hq, hk) for sh in shapes)
+    W.ws = torch.empty(max(W.ws_bytes, 256), dtype=torch.uint8, device=dev)
     # one set of plan buffers per iteration: a later iteration never
     # overwrites host memory whose copy may still be queued
     W.tables_dev = [torch.empty((1, 4096), dtype=torch.int32, device=dev) for _ in range(2)]
@@ -176,7 +179,8 @@ def _low_step(torch, ppas, W, stream, timers=None, host=None):
                     e0 = torch.cuda.Event(enable_timing=True)
                     e0.record(stream)
                 ppas.ppas_attention_step(q, W.k_cache[layer], W.v_cache[layer], W.nb, tables, width, st.q_len,
-                                         st.ctx_len, hq, hk, D, geo.scale, out, False, None, 0, W.err, stream)
+                                         st.ctx_len, hq, hk, D, geo.scale, out, False, W.ws, W.ws_bytes, W.err,
+                                         stream)
                 if timers is not None:
                     e1 = torch.cuda.Event(enable_timing=True)
                     e1.record(stream)

@@ -221,10 +221,8 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
         // cutting units evens the CTAs out at the cost of partials and a
         // merge; it is taken when it shortens the launch by more than that
         const int32_t nc = static_cast<int32_t>(std::min<int64_t>(n_ctas, tiles));
-        const int64_t cut_span = (total + static_cast<int64_t>(nc - 1) * kPrefillItemCost + nc - 1) / nc;
-        const bool cut = allow_split && cut_span + kPrefillMergeCost < whole_span;
         std::vector<std::vector<PrefillWork>> per_cta;
-        if (cut) {
+        if (allow_split) {
             per_cta.resize(nc);
             // stream-K: CTA c gets the cost range [total c / nc, total (c + 1) / nc)
             // of the units laid end to end; a unit is cut where a range ends,
@@ -258,6 +256,17 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
                     for (auto &pc : pieces) pc.second.part = static_cast<uint16_t>(lp.n_part++);
                 }
                 for (auto &pc : pieces) per_cta[pc.first].push_back(pc.second);
+            }
+            int64_t cut_span = 0;
+            for (const auto &v : per_cta) {
+                int64_t load = 0;
+                for (const PrefillWork &w : v) load += w.kt1 - w.kt0 + kPrefillItemCost;
+                cut_span = std::max(cut_span, load);
+            }
+            if (lp.n_part == 0 || cut_span + kPrefillMergeCost >= whole_span) {
+                per_cta = std::move(whole);  // not worth the partials
+                lp.split_units.clear();
+                lp.n_part = 0;
             }
         } else {
             per_cta = std::move(whole);

@@ -37,7 +37,7 @@ constexpr int kMaxPrefillWork = 2400;   // items per launch (bounded by the 32 K
 constexpr int kMaxPrefillCtas = 256;    // CTAs per launch (one per SM)
 constexpr int kPrefillItemCost = 3;     // per-item overhead (Q load, pipeline fill, epilogue), in KV tiles
 constexpr int kPrefillMinPiece = 4;     // shortest piece of a split unit, in KV tiles
-constexpr int kPrefillMergeCost = 4;    // partial writes and the merge launch, in KV tiles
+constexpr int kPrefillMergeCost = 6;    // partial writes and the merge launch, in KV tiles
 constexpr uint16_t kNoPart = 0xFFFF;    // an item of an unsplit unit
 
 struct PrefillSeq {

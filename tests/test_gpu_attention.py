@@ -237,7 +237,7 @@ def test_full_size_sampled_rows(ppas, name, geo, mk):
 
 def test_split_kv_and_unsplit_fallback_agree(ppas):
     """A chunk over a long prefix runs split over its KV range (partials merged
-    by the last CTA); with a workspace too small for the partials the same
+    by the merge kernel); with a workspace too small for the partials the same
     step runs unsplit.  Both match the oracle."""
     geo = QWEN
     shape = wl.StepShape([1, 300, 130], [9000, 12000, 7000])
@@ -255,3 +255,30 @@ def test_split_kv_and_unsplit_fallback_agree(ppas):
         assert_close(host64(out), want, f"workspace {ws_bytes}")
         outs.append(out)
     assert full > 1 << 20
+
+
+def _many_short_chunks():
+    # 130 prefill chunks (more than one launch holds) plus 3 decode rows
+    rng = np.random.default_rng(5)
+    q = [int(x) for x in rng.integers(2, 300, size=130)] + [1, 1, 1]
+    p = [int(x) for x in rng.integers(0, 3000, size=130)] + [4000, 5000, 6000]
+    return wl.StepShape(q, [a + b for a, b in zip(q, p)])
+
+
+MULTI = [
+    ("130 chunks + 3 decodes", QWEN, _many_short_chunks),
+    # 157 query tiles x 16 head slots: more items than one launch holds
+    ("one 20000-token chunk", LLAMA, lambda: wl.StepShape([20000], [20500])),
+]
+
+
+@pytest.mark.parametrize("name,geo,mk", MULTI, ids=[m[0] for m in MULTI])
+def test_steps_planned_over_several_launches(ppas, name, geo, mk):
+    shape = mk()
+    c = device_case(geo, shape, seed=9, extra_blocks=16, nan_fill=True)
+    out = run_step(ppas, c, False)
+    torch.cuda.synchronize()
+    o = out.float().cpu().numpy()
+    rows = sample_rows(shape, geo.n_q_heads, 4 if len(shape.q_lens) > 10 else 256, seed=2)
+    got = o[[r for r, _ in rows], [h for _, h in rows]]
+    assert_close(got, oracle_rows(c, rows), name)
