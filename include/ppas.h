@@ -191,6 +191,16 @@ size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
                                      const int32_t *h_ctx_lens, int32_t n_q_heads,
                                      int32_t n_kv_heads);
 
+/* ---------------------------------------------------------------------------
+ * Number of kernels ppas_attention_step launches for this step when given a
+ * workspace of workspace_bytes (host only, no CUDA call): prefill launches,
+ * the merge launch after each prefill launch whose plan cuts units, and
+ * decode launches.  Memsets are not counted.  Returns -1 for arguments
+ * ppas_attention_step would reject (see there); 0 for n_seqs == 0.
+ * ------------------------------------------------------------------------- */
+int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
+                                    int32_t n_q_heads, int32_t n_kv_heads, size_t workspace_bytes);
+
 ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
                                 int32_t num_blocks, const int32_t *d_block_tables,
                                 int32_t max_blocks_per_seq, const int32_t *h_q_lens,

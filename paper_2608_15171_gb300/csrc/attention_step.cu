@@ -409,6 +409,29 @@ extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h
            plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas).total_bytes();
 }
 
+extern "C" int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
+                                               int32_t n_q_heads, int32_t n_kv_heads, size_t workspace_bytes) {
+    if (n_seqs < 0 || (n_seqs > 0 && (!h_q_lens || !h_ctx_lens))) return -1;
+    if (n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads) return -1;
+    const int32_t g = n_q_heads / n_kv_heads;
+    if (g != 1 && g != 2 && g != 4 && g != 8) return -1;
+    for (int32_t s = 0; s < n_seqs; ++s) {
+        if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return -1;
+        if (h_q_lens[s] > 1 && h_ctx_lens[s] > 65535 * kPrefillKT) return -1;
+    }
+    if (n_seqs == 0) return 0;
+    // the same plans as ppas_attention_step
+    const DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
+    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
+    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
+    if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
+        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false, n_ctas);
+    int32_t n = static_cast<int32_t>((dp.rows.size() + kMaxDecodeRows - 1) / kMaxDecodeRows);
+    for (const PrefillLaunchPlan &lp : pf.launches)
+        n += 1 + static_cast<int32_t>((lp.split_units.size() + kMaxMergeUnits - 1) / kMaxMergeUnits);
+    return n;
+}
+
 extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
                                            int32_t num_blocks, const int32_t *d_block_tables,
                                            int32_t max_blocks_per_seq, const int32_t *h_q_lens,

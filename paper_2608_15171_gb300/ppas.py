@@ -36,7 +36,7 @@ PPAS_REQ_PENDING, PPAS_REQ_WAITING, PPAS_REQ_RUNNING, PPAS_REQ_FINISHED = 0, 1, 
 EXPORTED = ("ppas_sched_create", "ppas_sched_destroy", "ppas_sched_free_blocks", "ppas_plan_step",
             "ppas_kv_append", "ppas_attention_workspace_size", "ppas_attention_step",
             "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc",
-            "ppas_debug_wait_timeout")
+            "ppas_debug_wait_timeout", "ppas_attention_kernel_count")
 PPAS_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
 
 
@@ -76,6 +76,8 @@ _lib.ppas_kv_append.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int3
 _lib.ppas_kv_append.restype = _c.c_int32
 _lib.ppas_attention_workspace_size.argtypes = [_c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32]
 _lib.ppas_attention_workspace_size.restype = _c.c_size_t
+_lib.ppas_attention_kernel_count.argtypes = [_c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_size_t]
+_lib.ppas_attention_kernel_count.restype = _c.c_int32
 _lib.ppas_attention_step.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p,
                                      _c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_int32, _c.c_int32,
                                      _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_size_t,
@@ -171,6 +173,15 @@ def ppas_attention_workspace_size(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: 
     ql, cl = _i32(q_lens), _i32(ctx_lens)
     return int(_lib.ppas_attention_workspace_size(int(ql.size), _p32(ql), _p32(cl), int(n_q_heads),
                                                   int(n_kv_heads)))
+
+
+def ppas_attention_kernel_count(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: int, workspace_bytes: int) -> int:
+    ql, cl = _i32(q_lens), _i32(ctx_lens)
+    n = int(_lib.ppas_attention_kernel_count(int(ql.size), _p32(ql), _p32(cl), int(n_q_heads), int(n_kv_heads),
+                                             int(workspace_bytes)))
+    if n < 0:
+        raise PpasError(PPAS_ERR_INVALID_ARG, "ppas_attention_kernel_count")
+    return n
 
 
 def ppas_attention_step(q, k_cache, v_cache, num_blocks: int, d_block_tables, max_blocks_per_seq: int,

@@ -91,3 +91,23 @@ def test_workspace_size_is_a_pure_function_of_lengths(ppas):
     # a chunk over a long prefix is split over its KV range: partials need room
     assert ppas.ppas_attention_workspace_size([512], [24000], 16, 2) > 0
     assert ppas.ppas_attention_workspace_size([], [], 16, 2) == 0
+
+
+def test_kernel_count_follows_the_plan(ppas):
+    from paper_2608_15171_gb300 import workloads as wl
+    # one prefill launch (whole units) for the 16k chunk with no prefix
+    it1, it2 = wl.low_pressure_steps()
+    assert ppas.ppas_attention_kernel_count(it1.q_lens, it1.ctx_lens, 16, 2, 0) == 1
+    # the chunk over a 16k prefix is cut into pieces when the workspace holds
+    # their partials: prefill launch + merge launch; without it, one launch
+    ws = ppas.ppas_attention_workspace_size(it2.q_lens, it2.ctx_lens, 16, 2)
+    assert ws > 0
+    assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, ws) == 2
+    assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, 0) == 1
+    # decode rows alone: one decode launch
+    assert ppas.ppas_attention_kernel_count([1, 1], [3000, 5000], 16, 2, 1 << 30) == 1
+    assert ppas.ppas_attention_kernel_count([], [], 16, 2, 0) == 0
+    with pytest.raises(ppas.PpasError):
+        ppas.ppas_attention_kernel_count([0], [5], 16, 2, 0)
+    with pytest.raises(ppas.PpasError):
+        ppas.ppas_attention_kernel_count([4], [8], 16, 3, 0)
