@@ -247,6 +247,50 @@ def _high_step(torch, ppas, W, stream, timers=None):
     return launches
 
 
+def _mbt_sweep(torch, ppas, geo, dev, stream, reps=10, warmup=3, n_sets=8):
+    """Attention time of one layer for a 16,384-token prompt processed as
+    chunks of each static MBT (1k ... 16k), summed over its chunks (chunk i
+    has prefix i * MBT): the kernel-level MBT sensitivity the paper measures
+    with eight 2k chunks against one 16k chunk.  ``n_sets`` distinct
+    buffer sets are cycled so that repeats do not find their inputs in L2."""
+    prompt = 16384
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    nb = wl.blocks_for(prompt)
+    perm = wl.page_permutation(nb, 7)
+    table = torch.from_numpy(np.asarray(perm[:nb], dtype=np.int32).reshape(1, nb)).to(dev)
+    sets = [(wl.bf16_normal((nb, hk, 16, D), 100 + i, dev), wl.bf16_normal((nb, hk, 16, D), 200 + i, dev),
+             wl.bf16_normal((prompt, hq, D), 300 + i, dev)) for i in range(n_sets)]
+    out = torch.empty((prompt, hq, D), dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    res = {}
+    for mbt in (1024, 2048, 4096, 8192, 16384):
+        chunks = [([mbt], [(i + 1) * mbt]) for i in range(prompt // mbt)]
+        ws_bytes = max(ppas.ppas_attention_workspace_size(q, c, hq, hk) for q, c in chunks)
+        ws = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
+        total = 0.0
+        for i, (ql, cl) in enumerate(chunks):
+            t0 = i * mbt
+            times = []
+            for r in range(warmup + reps):
+                kc, vc, q = sets[r % n_sets]
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                ppas.ppas_attention_step(q[t0:t0 + mbt], kc, vc, nb, table, nb, ql, cl, hq, hk, D, geo.scale,
+                                         out[t0:t0 + mbt], False, ws, ws_bytes, err, stream)
+                e1.record(stream)
+                times.append((e0, e1))
+            torch.cuda.synchronize()
+            ts = sorted(a.elapsed_time(b) for a, b in times[warmup:])
+            total += ts[len(ts) // 2] * 1e3
+        res[str(mbt)] = round(total, 1)
+    assert err.item() == 0, f"device error flag {err.item()}"
+    return {"workload": "one layer's attention for a 16,384-token prompt (no prefix) chunked at each static MBT, "
+                        "Qwen2.5-3B geometry; median of 10 per chunk, summed over chunks",
+            "unit": "us", "attention_us": res,
+            "ratio_to_16k": {k: round(v / res["16384"], 3) for k, v in res.items()}}
+
+
 def _roofline_time_us(shape, geo, peaks, sustained=True):
     tf = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"] * 1e12
     bw = peaks["hbm_gbs"] * 1e9
@@ -355,6 +399,7 @@ def run_ours(args, rank, world, dist):
         "tflops": round(wl.step_flops(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e12, 1),
         "hbm_gbs": round(wl.step_bytes(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e9, 1)}
     del H
+    mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
 
     line = {
         "metric": METRIC, "value": round(step_us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
@@ -381,6 +426,7 @@ def run_ours(args, rank, world, dist):
                 sum(t for it, t in per_launch if it == i) * 1e3 / args.steps / geo.n_layers, 1)
             for i, sh in enumerate(shapes)},
         "mbt2k": mbt2k,
+        "mbt_sweep": mbt_sweep,
         "e2e": e2e,
         "gpu_launches": launches // args.steps * args.steps,
         "clocks": clocks,

@@ -203,12 +203,14 @@ class Scheduler:
 
 
 def replay(reqs: List[Request], num_blocks: int, free_order, threshold=N_TH, mbt_hi=B_MAX,
-           mbt_lo=B_CAP, width=None, max_steps=100000):
+           mbt_lo=B_CAP, width=None, max_steps=100000, durations=None):
     """Run the planner until every request finished; returns ``[(now_us, Step)]``.
 
     The clock is a deterministic integer: each iteration with work advances it
-    by ``15000 + 27 * prefill_tokens`` us; with nothing runnable it jumps to
-    the next arrival.
+    by ``15000 + 27 * prefill_tokens`` us, or, when ``durations`` is given, by
+    the next logged step duration (integer us, one per iteration with work, in
+    order: a closed-loop run's measured step times); with nothing runnable it
+    jumps to the next arrival.
     """
     sched = Scheduler(num_blocks, free_order)
     now = 0
@@ -225,5 +227,8 @@ def replay(reqs: List[Request], num_blocks: int, free_order, threshold=N_TH, mbt
             now = max(now, min(pending))
             continue
         out.append((now, step))
-        now += STEP_BASE_US + STEP_US_PER_PREFILL_TOKEN * step.prefill_tokens
+        if durations is None:
+            now += STEP_BASE_US + STEP_US_PER_PREFILL_TOKEN * step.prefill_tokens
+        else:
+            now += int(durations[len(out) - 1])
     raise RuntimeError("replay did not finish")

@@ -89,3 +89,34 @@ def test_burst_replay_plans_appends_and_attention(ppas, rate):
     # the device cache equals the oracle's appends, bit for bit
     assert np.array_equal(k_cache.float().cpu().numpy(), k_host)
     assert np.array_equal(v_cache.float().cpu().numpy(), v_host)
+
+
+def test_closed_loop_with_measured_clock(ppas):
+    """The closed-loop replay executes every planned step on the GPU (2
+    layers) and advances the clock by its measured time; the oracle planner
+    driven by the logged durations reproduces every plan and start time, and
+    the request metrics are consistent with the step log."""
+    from paper_2608_15171_gb300 import serving
+    geo = wl.QWEN25_3B
+    specs = wl.poisson_burst(6, 40.0, seed=4, prompt=(3000, 9000), output=(2, 6))
+    nb = serving.blocks_needed(specs)
+    width = wl.blocks_for(max(s.prompt_len + s.output_len for s in specs))
+    ex = serving.StepExecutor(geo, 2, nb, max_tokens=4096 + 8, max_rows=8, max_blocks_per_seq=width)
+    order = wl.page_permutation(nb, 4)
+    res = serving.closed_loop(specs, ex, order, 2, 4096, 1024, record_plans=True)
+    durations = [s.duration_us for s in res.steps]
+    assert all(d > 0 for d in durations)
+    want = op.replay([op.Request(s.arrival_us, s.prompt_len, s.output_len) for s in specs], nb, order,
+                     mbt_hi=4096, mbt_lo=1024, width=width, durations=durations)
+    assert len(want) == len(res.plans)
+    for rec, st, (t, so) in zip(res.steps, res.plans, want):
+        assert rec.now_us == t
+        assert st.q_len.tolist() == so.q_len and st.ctx_len.tolist() == so.ctx_len
+        assert st.slot_mapping.tolist() == so.slot_mapping and st.b_prefill == so.b_prefill
+    s = res.summary
+    assert s["requests"] == len(specs) and s["steps"] == len(res.steps)
+    for sp, f, e in zip(specs, res.first_token_us, res.finish_us):
+        assert sp.arrival_us < f <= e
+    end = res.steps[-1].now_us + res.steps[-1].duration_us
+    assert max(res.finish_us) == end
+    assert s["makespan_s"] == pytest.approx((end - min(sp.arrival_us for sp in specs)) / 1e6)

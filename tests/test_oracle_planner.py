@@ -162,3 +162,34 @@ def test_bad_arguments():
         sched.plan_step([], 0, mbt_hi=100, mbt_lo=200)
     with pytest.raises(ValueError):
         op.Scheduler(3, [0, 0, 1])
+
+
+def test_replay_with_logged_durations():
+    """Durations equal to the clock rule reproduce the default replay; other
+    durations shift arrivals relative to the plan and still satisfy every
+    replay invariant."""
+    specs = wl.poisson_burst(8, 2.0, seed=3, prompt=(3000, 9000), output=(2, 6))
+    nb = sum(wl.blocks_for(s.prompt_len + s.output_len) for s in specs) + 8
+    order = wl.page_permutation(nb, 3)
+    mk = lambda: [op.Request(s.arrival_us, s.prompt_len, s.output_len) for s in specs]
+    ref = op.replay(mk(), nb, order, mbt_hi=4096, mbt_lo=1024)
+    rule = [op.STEP_BASE_US + op.STEP_US_PER_PREFILL_TOKEN * st.prefill_tokens for _, st in ref]
+    same = op.replay(mk(), nb, order, mbt_hi=4096, mbt_lo=1024, durations=rule)
+    assert [(t, st.q_len, st.ctx_len, st.slot_mapping) for t, st in same] == \
+           [(t, st.q_len, st.ctx_len, st.slot_mapping) for t, st in ref]
+    # a fast clock (every step 1 ms): every request still gets exactly its
+    # prompt and output_len - 1 decodes
+    reqs = mk()
+    fast = op.replay(reqs, nb, order, mbt_hi=4096, mbt_lo=1024, durations=[1000] * 100000)
+    times = [t for t, _ in fast]
+    assert all(b - a >= 1000 for a, b in zip(times, times[1:]))
+    pre = [0] * len(specs)
+    dec = [0] * len(specs)
+    for _, st in fast:
+        for r, i in enumerate(st.req_idx):
+            if r < st.n_decode:
+                dec[i] += 1
+            else:
+                pre[i] += st.q_len[r]
+    assert pre == [s.prompt_len for s in specs]
+    assert dec == [s.output_len - 1 for s in specs]
