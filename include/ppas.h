@@ -157,7 +157,7 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * Mixed-batch attention step (device).
  * One scheduler iteration's attention: prefill chunks attend causally to
  * their own paged KV prefix and decode rows attend to their whole context,
- * all in one call (Section 5.2: prefill and decode tokens of one iteration
+ * all in one call (Section 6.2: prefill and decode tokens of one iteration
  * run together).  For sequence s with q_s = h_q_lens[s] new tokens and
  * context ctx_s = h_ctx_lens[s] (the new tokens are the last q_s positions,
  * already appended to the cache), query token t sits at position

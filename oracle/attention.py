@@ -6,7 +6,7 @@ imports this module.
 What is computed
 ----------------
 The paper (Section 2, prefill stores keys/values in the KV cache and decode
-generates tokens one at a time; Section 5.2, prefill and decode tokens of
+generates tokens one at a time; Section 6.2, prefill and decode tokens of
 different requests are scheduled together in one iteration) fixes the shape
 of the work but defines no attention arithmetic.  The oracle therefore takes
 the plain definition of causal scaled dot-product attention and applies it to

@@ -14,7 +14,7 @@ Passages followed
 * Section 2: continuous batching with chunked prefill; the MBT budget is
   shared by prefill and decode work of one iteration; long prompts are split
   into chunks across iterations.
-* Section 6 (Sarathi-Serve, which vLLM's chunked prefill follows): ongoing
+* Section 7 (Sarathi-Serve, which vLLM's chunked prefill follows): ongoing
   decodes are scheduled first and the remaining budget is filled with
   prefill work.
 
@@ -49,7 +49,7 @@ B_MAX = 16384
 B_CAP = 2048
 
 # replay clock (reading of the paper; 27 us/token ~ 668.6 ms / 25k tokens of
-# whole-model prefill at MBT 16k in Table 2)
+# whole-model prefill at MBT 16k in the prefill table of Section 6.1)
 STEP_BASE_US = 15000
 STEP_US_PER_PREFILL_TOKEN = 27
 

@@ -15,7 +15,7 @@ arrival processes are given):
   give each sequence consecutive runs of that order.
 * Requests: Poisson arrivals (cumulative exponential gaps in integer
   microseconds from t = 0), prompt and output lengths uniform over inclusive
-  integer ranges (Section 4.1 lengths: prompts 20k-30k, outputs 16-64).
+  integer ranges (Section 4.2 lengths: prompts 20k-30k, outputs 16-64).
 """
 from __future__ import annotations
 
