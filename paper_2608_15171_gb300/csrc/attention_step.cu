@@ -126,12 +126,31 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
             total_pages += static_cast<int64_t>((ctx_lens[s] + kPage - 1) / kPage) * n_kv_heads;
         }
     if (d.rows.empty()) return d;
-    // each (row, kv-head) gets a share of about kDecodeTargetCtas CTAs in
-    // proportion to its pages, so one step stays within one wave
-    for (int32_t s : d.rows) {
+    // each (row, kv-head) gets a share of kDecodeTargetCtas CTAs in proportion
+    // to its pages (largest remainders first), so one step fills one wave
+    const size_t nr = d.rows.size();
+    std::vector<int64_t> shares(nr);
+    {
+        const int64_t per_head = std::max<int64_t>(1, kDecodeTargetCtas / n_kv_heads);
+        int64_t given = 0;
+        std::vector<std::pair<int64_t, size_t>> rem(nr);  // (remainder, row)
+        for (size_t k = 0; k < nr; ++k) {
+            const int64_t pages = (ctx_lens[d.rows[k]] + kPage - 1) / kPage;
+            const int64_t num = per_head * pages * n_kv_heads;  // share = num / total_pages
+            shares[k] = num / total_pages;
+            rem[k] = {num % total_pages, k};
+            given += shares[k];
+        }
+        std::stable_sort(rem.begin(), rem.end(),
+                         [](const std::pair<int64_t, size_t> &a, const std::pair<int64_t, size_t> &b) {
+                             return a.first > b.first;
+                         });
+        for (size_t k = 0; k < nr && given < per_head; ++k, ++given) ++shares[rem[k].second];
+    }
+    for (size_t k = 0; k < nr; ++k) {
+        const int32_t s = d.rows[k];
         const int64_t pages = (ctx_lens[s] + kPage - 1) / kPage;
-        int64_t share = kDecodeTargetCtas * pages * n_kv_heads / total_pages / n_kv_heads;
-        share = std::max<int64_t>(share, 1);
+        const int64_t share = std::max<int64_t>(shares[k], 1);
         int64_t pps = (pages + share - 1) / share;
         pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
         pps = (pps + kDecodeWarps - 1) / kDecodeWarps * kDecodeWarps;
