@@ -14,6 +14,9 @@ Contents
     dot-product attention restricted to each query's causal prefix), written
     as un-page -> dense scores -> explicit mask -> max-subtracted softmax ->
     weighted sum of values.
+``oracle.mlp``
+    The gate-up projection of the decoder MLP profiled beside attention in
+    Section 6.1: ``silu(X W_gate^T) * (X W_up^T)`` in float64.
 ``oracle.planner``
     The P-PAS step planner: Algorithm 1 (pressure test and prefill budget),
     chunked-prefill step composition under the unchanged global budget
