@@ -291,6 +291,42 @@ def _mbt_sweep(torch, ppas, geo, dev, stream, reps=10, warmup=3, n_sets=8):
             "ratio_to_16k": {k: round(v / res["16384"], 3) for k, v in res.items()}}
 
 
+def _gateup_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3):
+    """The gate-up projection with the fused gated activation for a
+    16,384-token prompt of the Qwen2.5-3B MLP (hidden 2048, intermediate
+    11008): one 16k chunk against eight 2k chunks (Section 6.1)."""
+    T, H, I = 16384, 2048, 11008
+    x = wl.bf16_normal((T, H), 41, dev)
+    w = (wl.bf16_normal((2 * I, H), 42, dev).float() / math.sqrt(H)).to(torch.bfloat16)
+    wp = torch.empty_like(w)
+    ppas.ppas_gateup_pack(w, wp, H, I, stream)
+    y = torch.empty((T, I), dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    res = {}
+    for name, chunk in (("16k", 16384), ("2k", 2048)):
+        times = []
+        for r in range(warmup + reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for c in range(0, T, chunk):
+                ppas.ppas_gateup_swiglu(x[c:c + chunk], wp, y[c:c + chunk], chunk, H, I, err, stream)
+            e1.record(stream)
+            times.append((e0, e1))
+        torch.cuda.synchronize()
+        ts = sorted(a.elapsed_time(b) for a, b in times[warmup:])
+        res[name] = ts[len(ts) // 2] * 1e3
+    assert err.item() == 0, f"device error flag {err.item()}"
+    flops = 2.0 * T * H * 2 * I
+    peak = peaks["bf16_tflops"]
+    return {"workload": "gate-up projection + silu*up, 16,384 tokens, hidden 2048, intermediate 11008, bf16",
+            "kernel": "gateup_swiglu_kernel", "unit": "us",
+            "one_16k_chunk_us": round(res["16k"], 1), "eight_2k_chunks_us": round(res["2k"], 1),
+            "ratio_2k_to_16k": round(res["2k"] / res["16k"], 3),
+            "tflops_16k": round(flops / (res["16k"] * 1e-6) / 1e12, 1),
+            "frac_16k_vs_burst_peak": round(flops / (res["16k"] * 1e-6) / 1e12 / peak, 4)}
+
+
 def _roofline_time_us(shape, geo, peaks, sustained=True):
     tf = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"] * 1e12
     bw = peaks["hbm_gbs"] * 1e9
@@ -400,6 +436,7 @@ def run_ours(args, rank, world, dist):
         "hbm_gbs": round(wl.step_bytes(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e9, 1)}
     del H
     mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
+    gateup = _gateup_bench(torch, ppas, dev, stream, peaks)
 
     line = {
         "metric": METRIC, "value": round(step_us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
@@ -427,6 +464,7 @@ def run_ours(args, rank, world, dist):
             for i, sh in enumerate(shapes)},
         "mbt2k": mbt2k,
         "mbt_sweep": mbt_sweep,
+        "gateup": gateup,
         "e2e": e2e,
         "gpu_launches": launches // args.steps * args.steps,
         "clocks": clocks,

@@ -210,6 +210,29 @@ ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *
                                 int32_t *d_err_flag, void *stream);
 
 /* ---------------------------------------------------------------------------
+ * Gate-up projection of the decoder MLP with the gated activation fused in
+ * (the GEMM Section 6.1 profiles beside attention):
+ *   y[t, i] = silu(x[t] . w[i]) * (x[t] . w[inter + i]),  silu(a) = a / (1 + e^-a)
+ * for the stacked weight w = [w_gate; w_up] of shape [2*inter, hidden].
+ *
+ * ppas_gateup_pack (device, async on `stream`): rearranges w (device bf16
+ *   [2*inter, hidden], gate rows then up rows) into w_packed (device bf16,
+ *   same size, caller-owned): block j of 256 rows holds gate rows
+ *   128j..128j+127 then up rows inter+128j..inter+128j+127.  Done once per
+ *   weight.
+ * ppas_gateup_swiglu (device, async on `stream`): x device bf16
+ *   [n_tokens, hidden] row-major, w_packed as produced above, y device bf16
+ *   [n_tokens, inter] row-major (caller-owned).  fp32 accumulation.
+ * Both: hidden a multiple of 64 and inter a multiple of 128, else
+ * PPAS_ERR_UNSUPPORTED; pointers 16-byte aligned, else PPAS_ERR_INVALID_ARG;
+ * n_tokens == 0 is a no-op.  d_err_flag (device int32 or NULL) records
+ * PPAS_DEVERR_TIMEOUT if a bounded wait runs out.
+ * ------------------------------------------------------------------------- */
+ppas_status ppas_gateup_pack(const void *w, void *w_packed, int32_t hidden, int32_t inter, void *stream);
+ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int32_t n_tokens, int32_t hidden,
+                               int32_t inter, int32_t *d_err_flag, void *stream);
+
+/* ---------------------------------------------------------------------------
  * Attention step without a caller-provided workspace.  The paper has no
  * counterpart to this entry point: it exists for callers that may not
  * allocate device memory at all (a serving loop that gave all of HBM to its

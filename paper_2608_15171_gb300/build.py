@@ -21,7 +21,7 @@ LIB_PATH = os.path.join(HERE, "libppas.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["planner.cpp", "attention_step.cu", "kv_append.cu", "attn_prefill.cu", "attn_decode.cu",
-           "attention_noalloc.cu"]
+           "attention_noalloc.cu", "gateup.cu"]
 
 
 def _nvcc() -> str:

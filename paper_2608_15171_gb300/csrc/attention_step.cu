@@ -100,6 +100,19 @@ bool encode_kv_map(CUtensorMap *map, const void *cache, int32_t num_blocks, int3
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                    uint32_t box_outer) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {inner * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Q [total_q, n_q_heads, 128] bf16: dims (column, head, token); one box =
 // 128 tokens of one head x 64 columns.
 bool encode_q_map(CUtensorMap *map, const void *q, int32_t total_q, int32_t n_q_heads) {
@@ -621,4 +634,34 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
             return PPAS_ERR_CUDA;
     }
     return PPAS_OK;
+}
+
+extern "C" ppas_status ppas_gateup_pack(const void *w, void *w_packed, int32_t hidden, int32_t inter, void *stream) {
+    if (hidden < 64 || hidden % 64 || inter < 128 || inter % 128) return PPAS_ERR_UNSUPPORTED;
+    if (!w || !w_packed || !aligned16(w) || !aligned16(w_packed)) return PPAS_ERR_INVALID_ARG;
+    return launch_gateup_pack(w, w_packed, hidden, inter, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? PPAS_OK
+               : PPAS_ERR_CUDA;
+}
+
+extern "C" ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int32_t n_tokens,
+                                          int32_t hidden, int32_t inter, int32_t *d_err_flag, void *stream) {
+    if (n_tokens < 0) return PPAS_ERR_INVALID_ARG;
+    if (hidden < 64 || hidden % 64 || inter < 128 || inter % 128) return PPAS_ERR_UNSUPPORTED;
+    if (n_tokens == 0) return PPAS_OK;
+    if (!x || !w_packed || !y || !aligned16(x) || !aligned16(w_packed) || !aligned16(y)) return PPAS_ERR_INVALID_ARG;
+    CUtensorMap tm_x, tm_w;
+    if (!encode_bf16_2d(&tm_x, x, static_cast<uint64_t>(hidden), static_cast<uint64_t>(n_tokens), 64, 128) ||
+        !encode_bf16_2d(&tm_w, w_packed, static_cast<uint64_t>(hidden), 2ull * inter, 64, 256))
+        return PPAS_ERR_CUDA;
+    GateUpParams gp;
+    gp.y = static_cast<__nv_bfloat16 *>(y);
+    gp.n_tokens = n_tokens;
+    gp.hidden = hidden;
+    gp.inter = inter;
+    gp.err = d_err_flag;
+    const int64_t tiles = static_cast<int64_t>((n_tokens + 127) / 128) * (inter / 128);
+    const int grid = static_cast<int>(std::min<int64_t>(tiles, device_sm_count()));
+    return launch_gateup(tm_x, tm_w, gp, grid, static_cast<cudaStream_t>(stream)) == cudaSuccess ? PPAS_OK
+                                                                                                  : PPAS_ERR_CUDA;
 }

@@ -193,6 +193,24 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
 
 int32_t device_sm_count();
 
+// ------------------------------------------------------------------ gate-up projection
+struct GateUpParams {
+    __nv_bfloat16 *y;  // [n_tokens, inter]
+    int32_t n_tokens;
+    int32_t hidden;    // multiple of 64
+    int32_t inter;     // multiple of 128
+    int32_t *err;
+};
+
+// 2D bf16 row-major tensor [outer, inner] with a (box_inner x box_outer) box,
+// 128-byte swizzle (box_inner * 2 bytes must be 128)
+bool encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+                    uint32_t box_outer);
+
+cudaError_t launch_gateup(const CUtensorMap &tm_x, const CUtensorMap &tm_w, const GateUpParams &p, int grid,
+                          cudaStream_t st);
+cudaError_t launch_gateup_pack(const void *w, void *wp, int hidden, int inter, cudaStream_t st);
+
 // launchers (return a cudaError_t of the launch)
 cudaError_t launch_wait_timeout(int32_t *err, unsigned long long limit_ns, cudaStream_t st);
 

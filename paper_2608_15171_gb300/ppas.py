@@ -36,7 +36,8 @@ PPAS_REQ_PENDING, PPAS_REQ_WAITING, PPAS_REQ_RUNNING, PPAS_REQ_FINISHED = 0, 1, 
 EXPORTED = ("ppas_sched_create", "ppas_sched_destroy", "ppas_sched_free_blocks", "ppas_plan_step",
             "ppas_kv_append", "ppas_attention_workspace_size", "ppas_attention_step",
             "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc",
-            "ppas_debug_wait_timeout", "ppas_attention_kernel_count")
+            "ppas_debug_wait_timeout", "ppas_attention_kernel_count", "ppas_gateup_pack",
+            "ppas_gateup_swiglu")
 PPAS_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
 
 
@@ -78,6 +79,11 @@ _lib.ppas_attention_workspace_size.argtypes = [_c.c_int32, _P32, _P32, _c.c_int3
 _lib.ppas_attention_workspace_size.restype = _c.c_size_t
 _lib.ppas_attention_kernel_count.argtypes = [_c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_size_t]
 _lib.ppas_attention_kernel_count.restype = _c.c_int32
+_lib.ppas_gateup_pack.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32, _c.c_void_p]
+_lib.ppas_gateup_pack.restype = _c.c_int32
+_lib.ppas_gateup_swiglu.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32, _c.c_int32,
+                                    _c.c_void_p, _c.c_void_p]
+_lib.ppas_gateup_swiglu.restype = _c.c_int32
 _lib.ppas_attention_step.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p,
                                      _c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_int32, _c.c_int32,
                                      _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_size_t,
@@ -173,6 +179,17 @@ def ppas_attention_workspace_size(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: 
     ql, cl = _i32(q_lens), _i32(ctx_lens)
     return int(_lib.ppas_attention_workspace_size(int(ql.size), _p32(ql), _p32(cl), int(n_q_heads),
                                                   int(n_kv_heads)))
+
+
+def ppas_gateup_pack(w, w_packed, hidden: int, inter: int, stream=None) -> None:
+    _check(_lib.ppas_gateup_pack(_ptr(w), _ptr(w_packed), int(hidden), int(inter), _stream(stream)),
+           "ppas_gateup_pack")
+
+
+def ppas_gateup_swiglu(x, w_packed, y, n_tokens: int, hidden: int, inter: int, d_err_flag=None,
+                       stream=None) -> None:
+    _check(_lib.ppas_gateup_swiglu(_ptr(x), _ptr(w_packed), _ptr(y), int(n_tokens), int(hidden), int(inter),
+                                   _ptr(d_err_flag), _stream(stream)), "ppas_gateup_swiglu")
 
 
 def ppas_attention_kernel_count(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: int, workspace_bytes: int) -> int:

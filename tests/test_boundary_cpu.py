@@ -111,3 +111,25 @@ def test_kernel_count_follows_the_plan(ppas):
         ppas.ppas_attention_kernel_count([0], [5], 16, 2, 0)
     with pytest.raises(ppas.PpasError):
         ppas.ppas_attention_kernel_count([4], [8], 16, 3, 0)
+
+
+def test_gateup_argument_errors_before_device_work(ppas):
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_swiglu(16, 16, 16, 4, 100, 256, None, 0)   # hidden not a multiple of 64
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_swiglu(16, 16, 16, 4, 128, 200, None, 0)   # inter not a multiple of 128
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_swiglu(0, 16, 16, 4, 128, 256, None, 0)    # null input
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_swiglu(16, 16, 16, -1, 128, 256, None, 0)
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    ppas.ppas_gateup_swiglu(16, 16, 16, 0, 128, 256, None, 0)       # no tokens: no-op
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_pack(16, 16, 64, 100, 0)
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    with pytest.raises(ppas.PpasError) as e:
+        ppas.ppas_gateup_pack(8, 16, 64, 128, 0)                     # misaligned
+    assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
