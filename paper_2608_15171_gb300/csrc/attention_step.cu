@@ -164,9 +164,9 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
         const int32_t s = d.rows[k];
         const int64_t pages = (ctx_lens[s] + kPage - 1) / kPage;
         const int64_t share = std::max<int64_t>(shares[k], 1);
+        // even splits (the last one short by fewer than n_splits pages)
         int64_t pps = (pages + share - 1) / share;
         pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
-        pps = (pps + kDecodeWarps - 1) / kDecodeWarps * kDecodeWarps;
         pps = std::min<int64_t>(pps, kDecodeMaxPagesPerSplit);
         const int32_t ns = static_cast<int32_t>((pages + pps - 1) / pps);
         d.n_splits.push_back(ns);

@@ -278,15 +278,37 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     __threadfence();
     for (int hh = tid / kHeadDim; hh < g; hh += hstep) {
         const int head = kvh * g + hh;
-        float M = -INFINITY;
-        for (int s = 0; s < row.n_splits; ++s)
-            M = fmaxf(M, __ldcg(p.part_ml + (static_cast<int64_t>(row.part_base + s) * p.n_q_heads + head) * 2));
-        float L = 0.f, O = 0.f;
-        for (int s = 0; s < row.n_splits; ++s) {
-            const int64_t pi = static_cast<int64_t>(row.part_base + s) * p.n_q_heads + head;
-            const float f = ex2(__ldcg(p.part_ml + pi * 2) - M);
-            L += f * __ldcg(p.part_ml + pi * 2 + 1);
-            O += f * __ldcg(p.part_o + pi * kHeadDim + t);
+        // eight splits per round: their loads are independent and overlap
+        // (a serial chain of dependent loads here was the kernel's tail)
+        float M = -INFINITY, L = 0.f, O = 0.f;
+        for (int s0 = 0; s0 < row.n_splits; s0 += 8) {
+            float mv[8], lv[8], ov[8];
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                mv[k] = -INFINITY;
+                lv[k] = ov[k] = 0.f;
+                if (s0 + k < row.n_splits) {
+                    const int64_t pi = static_cast<int64_t>(row.part_base + s0 + k) * p.n_q_heads + head;
+                    const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + pi * 2));
+                    mv[k] = ml.x;
+                    lv[k] = ml.y;
+                    ov[k] = __ldcg(p.part_o + pi * kHeadDim + t);
+                }
+            }
+            float mr = M;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) mr = fmaxf(mr, mv[k]);
+            // rescale what the earlier rounds summed to the new maximum
+            const float a = M == -INFINITY ? 0.f : ex2(M - mr);
+            L *= a;
+            O *= a;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const float f = mv[k] == -INFINITY ? 0.f : ex2(mv[k] - mr);
+                L += f * lv[k];
+                O += f * ov[k];
+            }
+            M = mr;
         }
         const int64_t oi = (static_cast<int64_t>(row.q_row) * p.n_q_heads + head) * kHeadDim + t;
         if (p.out_fp32) static_cast<float *>(p.out)[oi] = O / L;
