@@ -327,7 +327,7 @@ def _gateup_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3):
             "frac_16k_vs_burst_peak": round(flops / (res["16k"] * 1e-6) / 1e12 / peak, 4)}
 
 
-def _roofline_time_us(shape, geo, peaks, sustained=True):
+def _roofline_time_us(shape, geo, peaks, sustained):
     tf = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"] * 1e12
     bw = peaks["hbm_gbs"] * 1e9
     return max(wl.step_flops(shape, geo) / tf, wl.step_bytes(shape, geo) / bw) * 1e6
@@ -398,7 +398,9 @@ def run_ours(args, rank, world, dist):
     attn_flops_per_launch = wl.step_flops(shapes[0], geo)
     achieved = attn_flops_per_launch / (avg_launch_ms * 1e-3) / 1e12
     peak = peaks["bf16_tflops_sustained"]
-    roof_step_us = sum(_roofline_time_us(sh, geo, peaks) for sh in shapes) * geo.n_layers
+    # the step roofline of the metric: max(FLOPs / burst bf16 peak, bytes / HBM)
+    roof_step_us = sum(_roofline_time_us(sh, geo, peaks, False) for sh in shapes) * geo.n_layers
+    roof_step_sus_us = sum(_roofline_time_us(sh, geo, peaks, True) for sh in shapes) * geo.n_layers
     step_us = ms * 1e3 / args.steps
     traffic = PREFILL_TRAFFIC.get(_src_hash("attn_prefill.cu"))
 
@@ -424,14 +426,17 @@ def run_ours(args, rank, world, dist):
         torch, dist, lambda tm: _high_step(torch, ppas, H, stream, tm), args.steps, args.warmup, stream, rank, False)
     assert H.err.item() == 0, f"device error flag {H.err.item()}"
     hs_us = ms_h * 1e3 / args.steps
-    roof_h_us = _roofline_time_us(H.shape, geo, peaks) * geo.n_layers
+    roof_h_us = _roofline_time_us(H.shape, geo, peaks, False) * geo.n_layers
+    roof_h_sus_us = _roofline_time_us(H.shape, geo, peaks, True) * geo.n_layers
     attn_h_ms = sum(a.elapsed_time(b) for _, a, b in timers_h) / args.steps
     mbt2k = {
         "workload": "MBT 2048: 4x512 chunks, prefixes ~U[0,24576) + 8 decodes ctx ~U[25000,25032), 36 layers",
         "q_lens": H.shape.q_lens, "ctx_lens": H.shape.ctx_lens,
         "step_us": round(hs_us, 1), "attention_us_per_layer": round(attn_h_ms * 1e3 / geo.n_layers, 2),
-        "roofline_us": round(roof_h_us, 1), "frac": round(roof_h_us / hs_us, 4),
+        "roofline_us": round(roof_h_us, 1), "peak_kind": f"{peaks_kind} burst bf16 and HBM copy",
+        "frac": round(roof_h_us / hs_us, 4),
         "frac_attention_only": round(roof_h_us / (attn_h_ms * 1e3), 4),
+        "frac_vs_sustained_peak": round(roof_h_sus_us / hs_us, 4),
         "tflops": round(wl.step_flops(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e12, 1),
         "hbm_gbs": round(wl.step_bytes(H.shape, geo) * geo.n_layers / (hs_us * 1e-6) / 1e9, 1)}
     del H
@@ -454,10 +459,9 @@ def run_ours(args, rank, world, dist):
                      "peak_kind": f"{peaks_kind} sustained bf16", "traffic": traffic,
                      "avg_launch_us": round(avg_launch_ms * 1e3, 1),
                      "flops_per_launch": attn_flops_per_launch},
-        "step_roofline": {"roofline_us": round(roof_step_us, 1), "frac": round(roof_step_us / step_us, 4),
-                          "frac_vs_burst_peak": round(
-                              sum(_roofline_time_us(sh, geo, peaks, False) for sh in shapes) * geo.n_layers
-                              / step_us, 4)},
+        "step_roofline": {"roofline_us": round(roof_step_us, 1), "peak_kind": f"{peaks_kind} burst bf16 and HBM copy",
+                          "frac": round(roof_step_us / step_us, 4),
+                          "frac_vs_sustained_peak": round(roof_step_sus_us / step_us, 4)},
         "per_iteration_us": {
             f"q={sh.q_lens[0]},p={sh.ctx_lens[0] - sh.q_lens[0]}": round(
                 sum(t for it, t in per_launch if it == i) * 1e3 / args.steps / geo.n_layers, 1)
