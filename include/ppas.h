@@ -148,6 +148,10 @@ ppas_status ppas_plan_step(ppas_sched *sched, ppas_request *reqs, int32_t n_reqs
  *   d_err_flag     : device int32 or NULL; PPAS_DEVERR_BAD_INDEX is written
  *                    when a slot is >= num_blocks*16 (that token is skipped)
  * head_dim must be a multiple of 8.  n_tokens == 0 is a no-op.
+ * PPAS_ERR_UNSUPPORTED when n_tokens * n_kv_heads * head_dim / 8 >= 2^31.
+ * The kernel is launched with programmatic stream serialization and lets the
+ * next kernel of the stream start its set-up early; an attention step that
+ * follows on the same stream still reads the cache only after it completes.
  * ------------------------------------------------------------------------- */
 ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *d_slot_mapping,
                            int32_t n_tokens, void *k_cache, void *v_cache, int32_t num_blocks,

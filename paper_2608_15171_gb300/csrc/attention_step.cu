@@ -425,6 +425,8 @@ extern "C" ppas_status ppas_kv_append(const void *k_new, const void *v_new, cons
     if (!k_new || !v_new || !d_slot_mapping || !k_cache || !v_cache) return PPAS_ERR_INVALID_ARG;
     if (!aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache))
         return PPAS_ERR_INVALID_ARG;
+    if (static_cast<int64_t>(n_tokens) * n_kv_heads * (head_dim / 8) >= (int64_t{1} << 31))
+        return PPAS_ERR_UNSUPPORTED;
     cudaError_t e = launch_kv_append(k_new, v_new, d_slot_mapping, n_tokens, k_cache, v_cache, num_blocks,
                                      n_kv_heads, head_dim, d_err_flag, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? PPAS_OK : PPAS_ERR_CUDA;

@@ -256,6 +256,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sg + kOffTmem);
+    // the set-up above overlaps the previous kernel of the stream; global
+    // memory (KV pages, Q, block tables, outputs) only after it has completed
+    grid_dep_wait();
 
     if (warp < 4) {
         // ------------------------------------------------------------ K/V producers
@@ -494,16 +497,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                     rb = add2(rb, make_float2(s[i + 2], s[i + 3]));
                 }
                 l_run = l_run * alpha + ((ra.x + ra.y) + (rb.x + rb.y));
-                if (jj >= 1 && __any_sync(0xffffffffu, need)) {
-#pragma unroll
-                    for (int c4 = 0; c4 < 4; ++c4) {
-                        float v[32];
-                        tmem_ld32_sync(t_o + c4 * 32, v);
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] *= alpha;
-                        tmem_st32_f(t_o + c4 * 32, v);
-                    }
-                }
                 if (j == last_j) {
                     // rows of the last page past the context may hold anything:
                     // zero them in V so that P = 0 times V stays 0.  Each tile's
@@ -530,6 +523,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                     for (int i = 0; i < 32; ++i) pk[i] = pack_bf16x2(s[64 * h + 2 * i], s[64 * h + 2 * i + 1]);
                     tmem_st32(t_s + 32 * h, pk);
+                }
+                if (jj >= 1 && __any_sync(0xffffffffu, need)) {
+#pragma unroll
+                    for (int c4 = 0; c4 < 4; ++c4) {
+                        float v[32];
+                        tmem_ld32_sync(t_o + c4 * 32, v);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] *= alpha;
+                        tmem_st32_f(t_o + c4 * 32, v);
+                    }
                 }
                 tmem_wait_st();
                 tc_fence_before();
@@ -575,7 +578,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int i = 0; i < 8; ++i)
                         __stcg(dst + i, make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]));
                 }
-                __stcg(reinterpret_cast<float2 *>(p.part_ml + (b * kTileQ + r) * 2), make_float2(m_used, l_run));
+                // two scalar stores: the paired float2 store costs the softmax loop
+                // register spills at its 200-register budget
+                __stcg(p.part_ml + (b * kTileQ + r) * 2, m_used);
+                __stcg(p.part_ml + (b * kTileQ + r) * 2 + 1, l_run);
             }
         }
         if (!ok) *abort_flag = 1;
@@ -597,6 +603,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // CTA (unit, head t, chunk c4, quarter) covers 32 rows x 32 columns, so a
 // warp reads 512 contiguous bytes of a partial chunk.
 __global__ void __launch_bounds__(256) prefill_merge_kernel(const __grid_constant__ MergeParams p) {
+    grid_dep_wait();  // the partials come from the prefill launch before this one
     const int hpc = p.heads_per_cta;
     const int lin = (blockIdx.x & 3) * 256 + threadIdx.x;  // 0..1023 within (unit, head, chunk)
     const int r = lin >> 3, j4 = lin & 7;
@@ -651,8 +658,8 @@ __global__ void __launch_bounds__(256) prefill_merge_kernel(const __grid_constan
 
 cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st) {
     if (p.n_units <= 0) return cudaSuccess;
-    prefill_merge_kernel<<<p.n_units * p.heads_per_cta * 16, 256, 0, st>>>(p);
-    return cudaGetLastError();
+    PdlLaunch l(dim3(p.n_units * p.heads_per_cta * 16), dim3(256), 0, st);
+    return cudaLaunchKernelEx(&l.cfg, prefill_merge_kernel, p);
 }
 
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
@@ -665,8 +672,8 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
         attr_set = true;
     }
     if (p.n_ctas <= 0) return cudaSuccess;
-    prefill_attn_kernel<<<p.n_ctas, kThreads, kSmemBytes, st>>>(tm_q, tm_k, tm_v, p);
-    return cudaGetLastError();
+    PdlLaunch l(dim3(p.n_ctas), dim3(kThreads), kSmemBytes, st);
+    return cudaLaunchKernelEx(&l.cfg, prefill_attn_kernel, tm_q, tm_k, tm_v, p);
 }
 
 }  // namespace ppas

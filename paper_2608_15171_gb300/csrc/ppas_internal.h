@@ -211,6 +211,25 @@ cudaError_t launch_gateup(const CUtensorMap &tm_x, const CUtensorMap &tm_w, cons
                           cudaStream_t st);
 cudaError_t launch_gateup_pack(const void *w, void *wp, int hidden, int inter, cudaStream_t st);
 
+// launch configuration with programmatic stream serialization: the kernel
+// may launch before its predecessor in the stream completes and orders its
+// own global accesses after it with grid_dep_wait()
+struct PdlLaunch {
+    cudaLaunchAttribute attr[1];
+    cudaLaunchConfig_t cfg;
+    PdlLaunch(dim3 grid, dim3 block, size_t smem, cudaStream_t st) {
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg = cudaLaunchConfig_t{};
+        cfg.gridDim = grid;
+        cfg.blockDim = block;
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = st;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+};
+
 // launchers (return a cudaError_t of the launch)
 cudaError_t launch_wait_timeout(int32_t *err, unsigned long long limit_ns, cudaStream_t st);
 

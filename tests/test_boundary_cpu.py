@@ -80,6 +80,9 @@ def test_kv_append_argument_errors(ppas):
     with pytest.raises(ppas.PpasError):
         ppas.ppas_kv_append(16, 16, 16, 3, 16, 16, 4, 2, 12, None, 0)
     ppas.ppas_kv_append(16, 16, 16, 0, 16, 16, 4, 2, 128, None, 0)  # no-op
+    # 2^27 tokens x 2 heads x 16 chunks = 2^32 elements: over the 32-bit index range
+    with pytest.raises(ppas.PpasError, match="UNSUPPORTED|unsupported"):
+        ppas.ppas_kv_append(16, 16, 16, 1 << 27, 16, 16, 4, 2, 128, None, 0)
 
 
 def test_workspace_size_is_a_pure_function_of_lengths(ppas):
