@@ -195,9 +195,12 @@ def improvement(ppas_values: Sequence[float], baseline_values: Sequence[float]) 
     return (1.0 - rm) * 100.0
 
 
-# the policies of Sections 4.3 and 5.1: P-PAS and the static budgets
+# the policies of Sections 4.3 and 5.1: P-PAS and the static budgets, plus
+# P-PAS with the strict reading of its threshold (more than two concurrent
+# prefills, N_p >= 3) as an ablation
 POLICIES = {"P-PAS": (2, 16384, 2048), "MBT 1k": (1 << 30, 1024, 1024), "MBT 2k": (1 << 30, 2048, 2048),
-            "MBT 4k": (1 << 30, 4096, 4096), "MBT 8k": (1 << 30, 8192, 8192), "MBT 16k": (1 << 30, 16384, 16384)}
+            "MBT 4k": (1 << 30, 4096, 4096), "MBT 8k": (1 << 30, 8192, 8192), "MBT 16k": (1 << 30, 16384, 16384),
+            "P-PAS N_th=3": (3, 16384, 2048)}
 
 
 def sweep(burst_rates, seeds, time_scale: float, policies=tuple(POLICIES), geo=wl.QWEN25_3B,

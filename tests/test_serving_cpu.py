@@ -38,6 +38,8 @@ def test_improvement_is_one_minus_geometric_mean_ratio():
 
 def test_policies_are_the_papers():
     assert serving.POLICIES["P-PAS"] == (2, 16384, 2048)
+    # the strict threshold reading (more than two prefills) as an ablation
+    assert serving.POLICIES["P-PAS N_th=3"] == (3, 16384, 2048)
     for name, (th, hi, lo) in serving.POLICIES.items():
-        if name != "P-PAS":
+        if not name.startswith("P-PAS"):
             assert hi == lo and th > 10**6
