@@ -170,6 +170,26 @@ def test_single_key_uniform_keys_constant_values(ppas):
     assert (out - 0.75).abs().max().item() <= 0.75 * 2.0 ** -8
 
 
+@pytest.mark.parametrize("growth", [0.2, 3.0])
+def test_scores_growing_along_the_context(ppas, growth):
+    """Keys of KV tile j (128 keys) scaled by 1 + growth * j, so every row's
+    scores grow along its context.  growth 0.2: the maximum from an item's
+    first tile stays in use and later exponentials exceed 1; growth 3: the
+    scores outgrow it by far more than 2^32 every few tiles, so the kernel
+    reads S again and raises the maximum (and rescales O) repeatedly.
+    Every element against the oracle."""
+    geo = QWEN
+    shape = wl.StepShape([1, 130, 1], [1500, 1700, 3000])
+    c = device_case(geo, shape, seed=31 + int(growth * 10))
+    for s_, ctx in enumerate(shape.ctx_lens):
+        for b in range(wl.blocks_for(ctx)):
+            c.k_cache[int(c.tables_np[s_, b])] *= 1.0 + growth * (b // 8)
+    out = run_step(ppas, c, True)
+    torch.cuda.synchronize()
+    assert torch.isfinite(out).all()
+    assert_close(host64(out), oracle_full(c), f"growth {growth}")
+
+
 def test_page_permutation_invariance_bitwise(ppas):
     geo = LLAMA
     shape = wl.StepShape([1, 1, 300], [2000, 77, 900])
