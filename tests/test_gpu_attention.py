@@ -173,11 +173,11 @@ def test_single_key_uniform_keys_constant_values(ppas):
 @pytest.mark.parametrize("growth", [0.2, 3.0])
 def test_scores_growing_along_the_context(ppas, growth):
     """Keys of KV tile j (128 keys) scaled by 1 + growth * j, so every row's
-    scores grow along its context.  growth 0.2: the maximum from an item's
-    first tile stays in use and later exponentials exceed 1; growth 3: the
-    scores outgrow it by far more than 2^32 every few tiles, so the kernel
-    reads S again and raises the maximum (and rescales O) repeatedly.
-    Every element against the oracle."""
+    scores grow along its context.  growth 0.2: the row maximum grows by less
+    than the kernel's 2^8 rescale threshold per tile, so a stale maximum stays
+    in use and later exponentials exceed 1; growth 3: it grows by far more on
+    almost every tile, so the maximum is raised and O rescaled in TMEM again
+    and again.  Every element against the oracle."""
     geo = QWEN
     shape = wl.StepShape([1, 130, 1], [1500, 1700, 3000])
     c = device_case(geo, shape, seed=31 + int(growth * 10))
