@@ -346,6 +346,35 @@ def _gateup_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3):
             "frac_16k_vs_burst_peak": round(flops / (res["16k"] * 1e-6) / 1e12 / peak, 4)}
 
 
+def _burst_replay(torch, ppas, geo, dev, peaks, rates=(0.5, 1.0, 2.0, 4.0), seed=0):
+    """The burst replay workload: a Poisson burst of 16 requests (prompts
+    ~U[20000, 30000], outputs ~U[16, 64]) at each rate, planned by the P-PAS
+    planner (threshold 2, MBT 16384 / 2048) and executed iteration by
+    iteration on all layers (appends + attention), the clock advanced by the
+    measured iteration times.  Per rate: iterations and device time under each
+    prefill budget with the time-weighted step-roofline fraction (burst
+    peak), and the requests' average latency."""
+    from paper_2608_15171_gb300 import serving
+    res = {}
+    for rate in rates:
+        specs = wl.poisson_burst(16, rate, seed)
+        nb = serving.blocks_needed(specs)
+        ex = serving.StepExecutor(geo, geo.n_layers, nb, max_tokens=16384 + len(specs), max_rows=len(specs) + 1,
+                                  max_blocks_per_seq=wl.blocks_for(max(s.prompt_len + s.output_len for s in specs)),
+                                  device=dev, seed=seed)
+        r = serving.closed_loop(specs, ex, wl.page_permutation(nb, seed), 2, 16384, 2048, record_plans=True)
+        reg = serving.roofline_by_regime(r, geo, geo.n_layers, peaks["bf16_tflops"], peaks["hbm_gbs"])
+        res[str(rate)] = {k: {"steps": v["steps"], "time_us": round(v["time_us"], 1),
+                              "roofline_us": round(v["roofline_us"], 1), "frac": round(v["frac"], 4)}
+                          for k, v in sorted(reg.items())}
+        res[str(rate)]["avg_latency_s"] = round(r.summary["avg_latency_s"], 4)
+        del ex
+        torch.cuda.empty_cache()
+    return {"workload": "Poisson burst of 16 requests, prompts ~U[20000,30000], outputs ~U[16,64], P-PAS threshold 2, "
+                        "MBT 16384/2048, every iteration on 36 layers (append + attention), closed loop",
+            "unit": "us", "rates_req_per_s": res}
+
+
 def _roofline_time_us(shape, geo, peaks, sustained):
     tf = peaks["bf16_tflops_sustained" if sustained else "bf16_tflops"] * 1e12
     bw = peaks["hbm_gbs"] * 1e9
@@ -468,6 +497,7 @@ def run_ours(args, rank, world, dist):
     del H
     mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
     gateup = _gateup_bench(torch, ppas, dev, stream, peaks)
+    burst = _burst_replay(torch, ppas, geo, dev, peaks)
 
     line = {
         "metric": METRIC, "value": round(step_us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
@@ -495,6 +525,7 @@ def run_ours(args, rank, world, dist):
         "mbt2k": mbt2k,
         "mbt_sweep": mbt_sweep,
         "gateup": gateup,
+        "burst_replay": burst,
         "e2e": e2e,
         "gpu_launches": launches // args.steps * args.steps,
         "clocks": clocks,

@@ -187,6 +187,29 @@ def summarize(res: RunResult) -> Dict[str, float]:
             "requests": len(res.specs)}
 
 
+def roofline_by_regime(res: RunResult, geo: wl.Geometry, n_layers: int, tflops: float,
+                       gbs: float) -> Dict[str, Dict[str, float]]:
+    """Time-weighted step-roofline fraction of a run recorded with its plans,
+    split by the prefill budget each iteration ran under (B_max or B_cap):
+    sum over its iterations of n_layers * max(FLOPs / tflops, bytes / gbs)
+    over the sum of their measured times (which also hold the appends and the
+    plan upload)."""
+    if len(res.plans) != len(res.steps):
+        raise ValueError("run was not recorded with its plans")
+    out: Dict[str, Dict[str, float]] = {}
+    for rec, st in zip(res.steps, res.plans):
+        shape = wl.StepShape([int(x) for x in st.q_len], [int(x) for x in st.ctx_len])
+        roof_us = n_layers * max(wl.step_flops(shape, geo) / (tflops * 1e12),
+                                 wl.step_bytes(shape, geo) / (gbs * 1e9)) * 1e6
+        d = out.setdefault(f"B={rec.b_prefill}", {"steps": 0, "time_us": 0.0, "roofline_us": 0.0})
+        d["steps"] += 1
+        d["time_us"] += rec.duration_us
+        d["roofline_us"] += roof_us
+    for d in out.values():
+        d["frac"] = d["roofline_us"] / d["time_us"]
+    return out
+
+
 def improvement(ppas_values: Sequence[float], baseline_values: Sequence[float]) -> float:
     """I_m of Section 5.1: (1 - R_m) x 100 %, R_m the geometric mean over the
     burst rates of P-PAS's value over the baseline's."""

@@ -2,6 +2,7 @@
 geometric-mean improvement I_m (Section 5.1), on hand-built runs."""
 import math
 
+import numpy as np
 import pytest
 
 from paper_2608_15171_gb300 import serving
@@ -43,3 +44,33 @@ def test_policies_are_the_papers():
     for name, (th, hi, lo) in serving.POLICIES.items():
         if not name.startswith("P-PAS"):
             assert hi == lo and th > 10**6
+
+
+def test_roofline_by_regime_sums_and_fractions():
+    """Two iterations under B_max and one under B_cap: per-regime sums of the
+    measured times and of n_layers x max(FLOPs / peak, bytes / bandwidth)."""
+    from types import SimpleNamespace
+    geo = wl.QWEN25_3B
+    shapes = [([16384], [16384]), ([8616], [25000]), ([1, 1, 512], [25000, 25001, 9000])]
+    budgets = [16384, 16384, 2048]
+    durations = [70000, 90000, 9000]
+    steps = [serving.StepRecord(0, d, 0, 1, 0, b, int(b == 2048)) for d, b in zip(durations, budgets)]
+    plans = [SimpleNamespace(q_len=np.array(q), ctx_len=np.array(c)) for q, c in shapes]
+    res = serving.RunResult(steps, [], [], [], plans=plans)
+    tf, bw = 1920.4, 6770.5
+    out = serving.roofline_by_regime(res, geo, 36, tf, bw)
+
+    def roof(q, c):
+        sh = wl.StepShape(q, c)
+        return 36 * max(wl.step_flops(sh, geo) / (tf * 1e12), wl.step_bytes(sh, geo) / (bw * 1e9)) * 1e6
+
+    hi = out["B=16384"]
+    assert hi["steps"] == 2 and hi["time_us"] == 160000
+    assert hi["roofline_us"] == pytest.approx(roof(*shapes[0]) + roof(*shapes[1]))
+    assert hi["frac"] == pytest.approx(hi["roofline_us"] / 160000)
+    lo = out["B=2048"]
+    assert lo["steps"] == 1 and lo["roofline_us"] == pytest.approx(roof(*shapes[2]))
+    # the 16k chunk's roofline is the tensor term: 572.6 us per layer
+    assert roof(*shapes[0]) / 36 == pytest.approx(572.6, abs=0.1)
+    with pytest.raises(ValueError):
+        serving.roofline_by_regime(serving.RunResult(steps, [], [], []), geo, 36, tf, bw)
