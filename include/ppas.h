@@ -190,6 +190,14 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * must lie in [0, num_blocks) for every position below ctx_len.
  * Rows with q_len == 1 run on the split-K decode kernel; longer rows run on
  * the tcgen05 prefill kernel.
+ * Stream semantics: all work is ordered after the work already on `stream`
+ * and everything later on `stream` is ordered after it, as for one kernel.
+ * Inside, when a step has both kinds of rows, the decode launch runs on a
+ * library-owned side stream forked from `stream` (an event) and joined back
+ * into it (a second event), so that it shares the GPU with the prefill
+ * launch; the prefill and merge kernels are launched with programmatic
+ * stream serialization (their set-up may overlap the kernel before them on
+ * `stream`; every global-memory access waits for that kernel to complete).
  * ------------------------------------------------------------------------- */
 size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
                                      const int32_t *h_ctx_lens, int32_t n_q_heads,
