@@ -255,40 +255,79 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
         const int32_t nc = static_cast<int32_t>(std::min<int64_t>(n_ctas, tiles));
         std::vector<std::vector<PrefillWork>> per_cta;
         if (allow_split) {
-            per_cta.resize(nc);
-            // stream-K: CTA c gets the cost range [total c / nc, total (c + 1) / nc)
-            // of the units laid end to end; a unit is cut where a range ends,
-            // and every cut adds one item's cost
-            total += static_cast<int64_t>(nc - 1) * kPrefillItemCost;
-            int32_t cta = 0;
-            int64_t pos = 0;  // cost handed out so far
-            for (size_t u = u0; u < u1; ++u) {
-                const Unit &un = units[u];
-                std::vector<std::pair<int32_t, PrefillWork>> pieces;  // (cta, item)
-                int32_t a = 0;
-                while (a < un.n_kt) {
-                    const int64_t end = total * (cta + 1) / nc;
-                    const int64_t room = end - pos - kPrefillItemCost;
-                    const int32_t left = un.n_kt - a;
-                    int32_t take = left;
-                    if (cta < nc - 1 && room < left) {
-                        if (room < kPrefillMinPiece) {  // too little left in this CTA's range
-                            ++cta;
-                            continue;
+            // stream-K with an even target: the units laid end to end in
+            // order are filled into CTAs up to a load T (tiles plus an item's
+            // cost per item), a unit cut where a CTA reaches T (no piece
+            // shorter than kPrefillMinPiece); T is the smallest load whose
+            // fill needs at most nc CTAs
+            auto fill = [&](int64_t T, std::vector<std::vector<std::pair<int32_t, PrefillWork>>> *out) -> int32_t {
+                int32_t cta = 0;
+                int64_t load = 0;
+                for (size_t u = u0; u < u1; ++u) {
+                    const Unit &un = units[u];
+                    int32_t a = 0;
+                    while (a < un.n_kt) {
+                        const int32_t left = un.n_kt - a;
+                        const int64_t room = T - load - kPrefillItemCost;
+                        int32_t take;
+                        if (left <= room) {
+                            take = left;
+                        } else {
+                            int64_t t = std::max<int64_t>(room, 0);
+                            if (left - t < kPrefillMinPiece) t = left - kPrefillMinPiece;
+                            if (t >= kPrefillMinPiece) {
+                                take = static_cast<int32_t>(t);
+                            } else if (load == 0) {
+                                // an empty CTA too small for a legal cut: the
+                                // remainder goes whole (or leaves a legal piece)
+                                take = left >= 2 * kPrefillMinPiece ? kPrefillMinPiece : left;
+                            } else {
+                                ++cta;  // nothing of this unit fits here
+                                load = 0;
+                                continue;
+                            }
                         }
-                        take = static_cast<int32_t>(room);
-                        if (left - take < kPrefillMinPiece) take = left;  // no sliver for the next CTA
+                        if (out) {
+                            if (static_cast<size_t>(cta) >= out->size()) out->resize(cta + 1);
+                            (*out)[cta].push_back({static_cast<int32_t>(u - u0), item(un, a, a + take)});
+                        }
+                        load += take + kPrefillItemCost;
+                        a += take;
+                        if (a < un.n_kt) {  // the unit goes on in the next CTA
+                            ++cta;
+                            load = 0;
+                        }
                     }
-                    pieces.push_back({cta, item(un, a, a + take)});
-                    pos += take + kPrefillItemCost;
-                    a += take;
                 }
-                if (pieces.size() > 1) {
-                    lp.split_units.push_back({un.seq, un.qt, un.slot, static_cast<int32_t>(pieces.size()), lp.n_part});
-                    for (auto &pc : pieces) pc.second.part = static_cast<uint16_t>(lp.n_part++);
-                }
-                for (auto &pc : pieces) per_cta[pc.first].push_back(pc.second);
+                return cta + (load > 0 ? 1 : 0);
+            };
+            int64_t lo = (total + nc - 1) / nc, hi = total;
+            while (lo < hi) {
+                const int64_t mid = lo + (hi - lo) / 2;
+                if (fill(mid, nullptr) <= nc) hi = mid; else lo = mid + 1;
             }
+            std::vector<std::vector<std::pair<int32_t, PrefillWork>>> filled;
+            fill(lo, &filled);
+            // pieces of a unit get consecutive partial slots
+            std::vector<int32_t> n_pieces(u1 - u0, 0);
+            for (const auto &v : filled)
+                for (const auto &pc : v) ++n_pieces[pc.first];
+            std::vector<int32_t> first_part(u1 - u0, -1), next_part(u1 - u0, 0);
+            for (size_t u = u0; u < u1; ++u) {
+                const int32_t k = static_cast<int32_t>(u - u0);
+                if (n_pieces[k] > 1) {
+                    first_part[k] = static_cast<int32_t>(lp.n_part);
+                    lp.split_units.push_back({units[u].seq, units[u].qt, units[u].slot, n_pieces[k], lp.n_part});
+                    lp.n_part += n_pieces[k];
+                }
+            }
+            per_cta.resize(filled.size());
+            for (size_t c = 0; c < filled.size(); ++c)
+                for (auto &pc : filled[c]) {
+                    if (first_part[pc.first] >= 0)
+                        pc.second.part = static_cast<uint16_t>(first_part[pc.first] + next_part[pc.first]++);
+                    per_cta[c].push_back(pc.second);
+                }
             int64_t cut_span = 0;
             for (const auto &v : per_cta) {
                 int64_t load = 0;
