@@ -8,7 +8,7 @@ import numpy as np
 import pytest
 import torch
 
-from _cases import (MAX_ABS, assert_close, device_case, host64, oracle_full, oracle_rows, run_step,
+from _cases import (MAX_ABS, assert_close, device_case, host32, host64, oracle_full, oracle_rows, run_step,
                     sample_rows)
 from oracle import attention as oa
 from paper_2608_15171_gb300 import workloads as wl
@@ -253,6 +253,21 @@ def test_full_size_sampled_rows(ppas, name, geo, mk):
     rows = sample_rows(shape, geo.n_q_heads, 96, seed=1)
     got = o[[r for r, _ in rows], [h for _, h in rows]]
     assert_close(got, oracle_rows(c, rows), name)
+
+
+@pytest.mark.parametrize("name,geo,mk", FULL, ids=[f[0] for f in FULL])
+def test_full_layer_every_element(ppas, name, geo, mk):
+    """One whole layer of every full-size workload, in the launch
+    configuration the benchmark times (whole units or stream-K pieces with
+    their merge, decode rows on the side stream): every output element
+    against the float64 oracle."""
+    shape = mk()
+    c = device_case(geo, shape, seed=2, extra_blocks=64)
+    out = run_step(ppas, c, False)
+    torch.cuda.synchronize()
+    want = oa.paged_attention(host64(c.q), host32(c.k_cache), host32(c.v_cache), c.tables_np, shape.q_lens,
+                              shape.ctx_lens, c.scale, workers=oa.default_workers())
+    assert_close(host64(out), want, name)
 
 
 def test_split_kv_and_unsplit_fallback_agree(ppas):
