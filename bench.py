@@ -215,7 +215,13 @@ def _low_step(torch, ppas, W, stream, timers=None, host=None):
 
 def _setup_high(torch, ppas, geo, dev, seed=0):
     """High-pressure workload: literal step, contexts pre-filled into pages."""
-    shape = wl.high_pressure_step(seed)
+    return _setup_step(torch, ppas, geo, wl.high_pressure_step(seed), dev, seed)
+
+
+def _setup_step(torch, ppas, geo, shape, dev, seed=0, n_sets=None):
+    """Buffers of a literal step for every layer: caches with every context
+    pre-filled, Q, new K/V, outputs; ``n_sets`` distinct sets cycled over
+    the layers (default one per layer)."""
     W = LayerSet()
     W.geo, W.shape = geo, shape
     need = sum(wl.blocks_for(c) for c in shape.ctx_lens)
@@ -232,7 +238,12 @@ def _setup_high(torch, ppas, geo, dev, seed=0):
     hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
     T = shape.total_q
     W.k_cache, W.v_cache, W.q, W.kn, W.vn, W.out = [], [], [], [], [], []
+    n_sets = geo.n_layers if n_sets is None else n_sets
     for layer in range(geo.n_layers):
+        if layer >= n_sets:
+            for lst in (W.k_cache, W.v_cache, W.q, W.kn, W.vn, W.out):
+                lst.append(lst[layer % n_sets])
+            continue
         s = 1000 * layer + seed + 500
         W.k_cache.append(wl.bf16_normal((W.nb, hk, 16, D), s + 1, dev))
         W.v_cache.append(wl.bf16_normal((W.nb, hk, 16, D), s + 2, dev))
@@ -344,6 +355,32 @@ def _gateup_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3):
             "ratio_2k_to_16k": round(res["2k"] / res["16k"], 3),
             "tflops_16k": round(flops / (res["16k"] * 1e-6) / 1e12, 1),
             "frac_16k_vs_burst_peak": round(flops / (res["16k"] * 1e-6) / 1e12 / peak, 4)}
+
+
+def _llama_bench(torch, ppas, dist, dev, stream, peaks, steps, warmup, rank):
+    """The Llama-3.1-8B-geometry steps (32q/8kv/d128, 32 layers), timed like
+    the MBT 2k step (append + attention per layer, no event between them):
+    MBT 16384 (one 16384 chunk + 4 decodes, ctx ~U[30000, 30064)) and MBT
+    2048 (chunks 683/683/682 over prefixes ~U[0, 30000 - q) + 16 decodes).
+    Four buffer sets cycle over the layers; each layer's K/V (0.5 to 2 GB)
+    is far larger than L2."""
+    geo = wl.LLAMA31_8B
+    res = {}
+    for name, mk in (("mbt16k", wl.llama_hi_step), ("mbt2k", wl.llama_lo_step)):
+        W = _setup_step(torch, ppas, geo, mk(0), dev, seed=3, n_sets=4)
+        ms, _, _, _ = _timed(torch, dist, lambda tm: _high_step(torch, ppas, W, stream), steps, warmup, stream,
+                             rank, False)
+        assert W.err.item() == 0, f"device error flag {W.err.item()}"
+        step_us = ms * 1e3 / steps
+        roof = _roofline_time_us(W.shape, geo, peaks, False) * geo.n_layers
+        roof_sus = _roofline_time_us(W.shape, geo, peaks, True) * geo.n_layers
+        res[name] = {"q_lens": W.shape.q_lens, "ctx_lens": W.shape.ctx_lens, "step_us": round(step_us, 1),
+                     "us_per_layer": round(step_us / geo.n_layers, 1), "roofline_us": round(roof, 1),
+                     "frac": round(roof / step_us, 4), "frac_vs_sustained_peak": round(roof_sus / step_us, 4)}
+        del W
+        torch.cuda.empty_cache()
+    return {"workload": "Llama-3.1-8B attention geometry 32q/8kv/d128, 32 layers, append + attention per layer",
+            "peak_kind": "measured burst bf16 and HBM copy", **res}
 
 
 def _burst_replay(torch, ppas, geo, dev, peaks, rates=(0.5, 1.0, 2.0, 4.0), seed=0):
@@ -497,6 +534,7 @@ def run_ours(args, rank, world, dist):
     del H
     mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
     gateup = _gateup_bench(torch, ppas, dev, stream, peaks)
+    llama = _llama_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     burst = _burst_replay(torch, ppas, geo, dev, peaks)
 
     line = {
@@ -525,6 +563,7 @@ def run_ours(args, rank, world, dist):
         "mbt2k": mbt2k,
         "mbt_sweep": mbt_sweep,
         "gateup": gateup,
+        "llama": llama,
         "burst_replay": burst,
         "e2e": e2e,
         "gpu_launches": launches // args.steps * args.steps,
@@ -576,7 +615,29 @@ def cpu_baseline(W, cache, torch, args):
     return {"value": round(us_per_step, 1), "unit": "us", "cores": workers, "kind": "oracle",
             "sample": f"{n} runs of the oracle on the last {rows} query tokens (all 16 heads) of the "
                       f"16384-token chunk over its full 16384-token context, {total_t:.1f} s, "
-                      f"extrapolated by causal pair count to the whole step (2 iterations x 36 layers)"}
+                      f"extrapolated by causal pair count to the whole step (2 iterations x 36 layers)",
+            "planner": _planner_timing()}
+
+
+def _planner_timing():
+    """Host planning of the burst replay (16 requests at 1 req/s, the
+    deterministic replay clock): the C++ planner through its binding against
+    the Python oracle planner, per planned iteration."""
+    from oracle import planner as op
+    from paper_2608_15171_gb300 import ppas
+    specs = wl.poisson_burst(16, 1.0, 0)
+    nb, width = 16 * 1879, 1900
+    order = wl.page_permutation(nb, 0)
+    t0 = time.perf_counter()
+    cpp = ppas.replay([(s.arrival_us, s.prompt_len, s.output_len) for s in specs], nb, order,
+                      cap_blocks_per_seq=width)
+    t1 = time.perf_counter()
+    ora = op.replay([op.Request(s.arrival_us, s.prompt_len, s.output_len) for s in specs], nb, order, width=width)
+    t2 = time.perf_counter()
+    assert len(cpp) == len(ora)
+    return {"workload": "burst replay, 16 requests at 1 req/s, P-PAS threshold 2, MBT 16384/2048",
+            "iterations": len(cpp), "cpp_us_per_iteration": round((t1 - t0) / len(cpp) * 1e6, 1),
+            "oracle_us_per_iteration": round((t2 - t1) / len(ora) * 1e6, 1)}
 
 
 def run_reference(args, rank, world):
