@@ -24,13 +24,20 @@
 //               one query row (its TMEM lane), loads its S row, masks by
 //               absolute position, runs the online softmax in fp32 (exp2
 //               domain) and stores P back to TMEM; at the end of an item it
-//               writes O (or a split's partial).
+//               writes O (or a piece's partial).  The two warpgroups take
+//               turns, tile 0 then tile 1, so that one tile's softmax runs
+//               under the other tile's MMAs.
 // Registers move from the producer/MMA warpgroups to the softmax warpgroups
 // with setmaxnreg.  The running max is only raised (and O rescaled in TMEM)
 // when it grows by more than 2^8; until then the stale max keeps every
 // exponent <= 2^8, and the final O / l is exact either way.
-// Long KV ranges may be split over several items (split-KV): each writes its
-// partial (m, l, O) and the last one of the tile to finish merges them.
+// The host plan may cut a long (query tile, head slot) unit into pieces on
+// consecutive CTAs (stream-K): each piece writes its partial (m, l, O) to the
+// workspace, and prefill_merge_kernel, launched after this kernel, combines
+// the pieces of every cut unit.
+// The kernel is launched with programmatic stream serialization: its set-up
+// (TMEM allocation, barriers, tensor-map prefetch) overlaps the kernel before
+// it on the stream, and global memory is touched only after grid_dep_wait().
 #include <math.h>
 
 #include "ppas_device.cuh"
