@@ -239,6 +239,9 @@ FULL = [
     ("high-pressure 4x512 + 8 decodes", QWEN, lambda: wl.high_pressure_step(0)),
     ("llama 16384 + 4 decodes", LLAMA, lambda: wl.llama_hi_step(0)),
     ("llama 3 chunks + 16 decodes", LLAMA, lambda: wl.llama_lo_step(0)),
+    # the decode rows of the Llama MBT 2k step alone (1.97 GB of K/V)
+    ("llama_decodes_only_16x30k", LLAMA,
+     lambda: wl.StepShape(wl.llama_lo_step(0).q_lens[:16], wl.llama_lo_step(0).ctx_lens[:16])),
 ]
 
 
