@@ -185,8 +185,8 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  *   d_err_flag    : device int32 or NULL (see PPAS_DEVERR_*)
  * Supported shapes: head_dim == 128, n_q_heads a multiple of n_kv_heads with
  * group size n_q_heads/n_kv_heads in {1, 2, 4, 8}, at most 256 q-heads
- * (512 with group >= 2), ctx_len <= 65535*128 for rows with q_len > 1;
- * otherwise PPAS_ERR_UNSUPPORTED.  n_seqs == 0 is a no-op.  Block ids in the tables
+ * (512 with group >= 2), ctx_len <= 65535*128 for rows with q_len > 1 and
+ * ctx_len <= 2^25 for rows with q_len == 1; otherwise PPAS_ERR_UNSUPPORTED.  n_seqs == 0 is a no-op.  Block ids in the tables
  * must lie in [0, num_blocks) for every position below ctx_len.
  * Rows with q_len == 1 run on the split-K decode kernel; longer rows run on
  * the tcgen05 prefill kernel.

@@ -416,6 +416,7 @@ ppas_status check_step(const void *q, const void *k_cache, const void *v_cache, 
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return PPAS_ERR_INVALID_ARG;
         // KV tile indices of the prefill items are 16-bit
         if (h_q_lens[s] > 1 && h_ctx_lens[s] > 65535 * kPrefillKT) return PPAS_ERR_UNSUPPORTED;
+        if (h_q_lens[s] == 1 && h_ctx_lens[s] > kMaxDecodeCtx) return PPAS_ERR_UNSUPPORTED;
         if (static_cast<int64_t>(h_ctx_lens[s]) > static_cast<int64_t>(max_blocks_per_seq) * kPage)
             return PPAS_ERR_INVALID_ARG;
         tq += h_q_lens[s];
@@ -491,6 +492,7 @@ extern "C" int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_
     for (int32_t s = 0; s < n_seqs; ++s) {
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return -1;
         if (h_q_lens[s] > 1 && h_ctx_lens[s] > 65535 * kPrefillKT) return -1;
+        if (h_q_lens[s] == 1 && h_ctx_lens[s] > kMaxDecodeCtx) return -1;
     }
     if (n_seqs == 0) return 0;
     // the same plans as ppas_attention_step

@@ -33,6 +33,8 @@ static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 // merge scratch (aliases the rings once every warp is done)
 constexpr int kMaxGroup = 8;
 static_assert(kDecodeWarps * kMaxGroup * (2 + kHeadDim) * 4 <= static_cast<int>(kOffBar), "merge scratch");
+static_assert(2 * kMaxDecodeSplitsPerRow * kMaxGroup * 4 <= static_cast<int>(kOffBar), "split weights");
+static_assert(kDecodeWarps >= kMaxGroup, "the split merge gives each head of a group one warp");
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -276,43 +278,66 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    for (int hh = tid / kHeadDim; hh < g; hh += hstep) {
-        const int head = kvh * g + hh;
-        // eight splits per round: their loads are independent and overlap
-        // (a serial chain of dependent loads here was the kernel's tail)
-        float M = -INFINITY, L = 0.f, O = 0.f;
-        for (int s0 = 0; s0 < row.n_splits; s0 += 8) {
-            float mv[8], lv[8], ov[8];
+    // Every split's (m, l) in one round of loads, turned into weights
+    // w = 2^(m - M) / L per (split, head); then each thread sums one head's
+    // 4 columns over the splits, 16 independent float4 loads at a time.
+    // (The rings are free: the weights live where they were.)
+    const int ns = row.n_splits;
+    float *sw = reinterpret_cast<float *>(sg);            // [ns][kMaxGroup] m, then w
+    float *sl = sw + kMaxDecodeSplitsPerRow * kMaxGroup;  // [ns][kMaxGroup] l
+    for (int i = tid; i < ns * g; i += blockDim.x) {
+        const int s_ = i / g, hh = i - s_ * g;
+        const int64_t pi = static_cast<int64_t>(row.part_base + s_) * p.n_q_heads + kvh * g + hh;
+        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + pi * 2));
+        sw[s_ * kMaxGroup + hh] = ml.x;
+        sl[s_ * kMaxGroup + hh] = ml.y;
+    }
+    __syncthreads();
+    const int hh = tid >> 5, c4 = tid & 31;  // warp hh: head hh; lane: 4 columns
+    if (hh < g) {
+        float M = -INFINITY, L = 0.f;
+        for (int s_ = lane; s_ < ns; s_ += 32) M = fmaxf(M, sw[s_ * kMaxGroup + hh]);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                mv[k] = -INFINITY;
-                lv[k] = ov[k] = 0.f;
-                if (s0 + k < row.n_splits) {
-                    const int64_t pi = static_cast<int64_t>(row.part_base + s0 + k) * p.n_q_heads + head;
-                    const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + pi * 2));
-                    mv[k] = ml.x;
-                    lv[k] = ml.y;
-                    ov[k] = __ldcg(p.part_o + pi * kHeadDim + t);
-                }
-            }
-            float mr = M;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) mr = fmaxf(mr, mv[k]);
-            // rescale what the earlier rounds summed to the new maximum
-            const float a = M == -INFINITY ? 0.f : ex2(M - mr);
-            L *= a;
-            O *= a;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const float f = mv[k] == -INFINITY ? 0.f : ex2(mv[k] - mr);
-                L += f * lv[k];
-                O += f * ov[k];
-            }
-            M = mr;
+        for (int o_ = 16; o_ >= 1; o_ >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o_));
+        for (int s_ = lane; s_ < ns; s_ += 32) {
+            const float m = sw[s_ * kMaxGroup + hh];
+            const float f = m == -INFINITY ? 0.f : ex2(m - M);
+            sw[s_ * kMaxGroup + hh] = f;
+            L += f * sl[s_ * kMaxGroup + hh];
         }
-        const int64_t oi = (static_cast<int64_t>(row.q_row) * p.n_q_heads + head) * kHeadDim + t;
-        if (p.out_fp32) static_cast<float *>(p.out)[oi] = O / L;
-        else static_cast<__nv_bfloat16 *>(p.out)[oi] = __float2bfloat16_rn(O / L);
+#pragma unroll
+        for (int o_ = 16; o_ >= 1; o_ >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o_);
+        const float inv_l = 1.f / L;
+        for (int s_ = lane; s_ < ns; s_ += 32) sw[s_ * kMaxGroup + hh] *= inv_l;
+    }
+    __syncthreads();
+    if (hh >= g) return;
+    const int head = kvh * g + hh;
+    const float4 *po = reinterpret_cast<const float4 *>(p.part_o) + c4;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s0 = 0; s0 < ns; s0 += 16) {
+        float4 ov[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            if (s0 + k < ns) {
+                const int64_t pi = static_cast<int64_t>(row.part_base + s0 + k) * p.n_q_heads + head;
+                ov[k] = __ldcg(po + pi * (kHeadDim / 4));
+            } else {
+                ov[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+            const float f = s0 + k < ns ? sw[(s0 + k) * kMaxGroup + hh] : 0.f;
+            acc = make_float4(acc.x + f * ov[k].x, acc.y + f * ov[k].y, acc.z + f * ov[k].z, acc.w + f * ov[k].w);
+        }
+    }
+    const int64_t oi = (static_cast<int64_t>(row.q_row) * p.n_q_heads + head) * kHeadDim + 4 * c4;
+    if (p.out_fp32) {
+        *reinterpret_cast<float4 *>(static_cast<float *>(p.out) + oi) = acc;
+    } else {
+        *reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.out) + oi) =
+            make_uint2(pack_bf16x2(acc.x, acc.y), pack_bf16x2(acc.z, acc.w));
     }
 }
 

@@ -141,6 +141,9 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
 constexpr int kDecodeWarps = 8;        // each warp streams its own pages (8 TMA issuers per SM)
 constexpr int kDecodeStages = 3;       // pages in flight per warp
 constexpr int kDecodeMaxPagesPerSplit = 1024;  // page ids of a split are staged in shared memory
+constexpr int kMaxDecodeSplitsPerRow = 2048;   // the merge keeps every split's weights in shared memory
+// longest decode context: kMaxDecodeSplitsPerRow splits of kDecodeMaxPagesPerSplit pages
+constexpr int64_t kMaxDecodeCtx = int64_t{kMaxDecodeSplitsPerRow} * kDecodeMaxPagesPerSplit * 16;
 constexpr int kMaxDecodeRows = 256;
 constexpr int kDecodeMinPagesPerSplit = 16;
 

@@ -70,6 +70,11 @@ def test_attention_argument_errors_before_device_work(ppas):
     with pytest.raises(E) as e:
         call(scale=-1.0)
     assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    # a decode row longer than 2^25 tokens (2048 splits of 1024 pages) is refused
+    big = (1 << 25) + 16
+    with pytest.raises(E) as e:
+        call(q_lens=[1], ctx_lens=[big], max_blocks_per_seq=big // 16 + 1)
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
     # empty step is a no-op
     call(q_lens=[], ctx_lens=[])
 
