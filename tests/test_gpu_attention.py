@@ -190,6 +190,43 @@ def test_scores_growing_along_the_context(ppas, growth):
     assert_close(host64(out), oracle_full(c), f"growth {growth}")
 
 
+def test_long_decode_rows(ppas):
+    """Decode rows far longer than the workloads': 2,097,157 tokens (129
+    splits of 1024 pages, merged in several rounds) against the oracle for
+    every head, and the longest row the boundary accepts, 2^25 tokens (2048
+    splits), with constant values, whose output is that constant whatever
+    the weights (up to the bf16 rounding of the weights)."""
+    geo = QWEN
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    shape = wl.StepShape([1], [(1 << 21) + 5])
+    c = device_case(geo, shape, seed=41, extra_blocks=3)
+    out = run_step(ppas, c, True)
+    torch.cuda.synchronize()
+    rows = [(0, h) for h in range(hq)]
+    assert_close(host64(out)[0], oracle_rows(c, rows), "2M-token decode row")
+    del c, out
+    torch.cuda.empty_cache()
+
+    ctx = 1 << 25
+    nb = wl.blocks_for(ctx)
+    k_cache = torch.empty((nb, hk, 16, D), dtype=torch.bfloat16, device="cuda")
+    step = 1 << 17
+    for b0 in range(0, nb, step):  # N(0,1) keys, drawn in slices to bound the float32 scratch
+        k_cache[b0:b0 + step] = wl.bf16_normal((min(step, nb - b0), hk, 16, D), 900 + b0 // step, "cuda")
+    v_cache = torch.full((nb, hk, 16, D), 0.75, dtype=torch.bfloat16, device="cuda")
+    tables = torch.from_numpy(wl.page_permutation(nb, 43).reshape(1, nb)).cuda()
+    q = wl.bf16_normal((1, hq, D), 44, "cuda")
+    out = torch.empty((1, hq, D), dtype=torch.float32, device="cuda")
+    ws_bytes = ppas.ppas_attention_workspace_size([1], [ctx], hq, hk)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ppas.ppas_attention_step(q, k_cache, v_cache, nb, tables, nb, [1], [ctx], hq, hk, D, geo.scale, out, True,
+                             ws, ws_bytes, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    assert (out - 0.75).abs().max().item() <= 0.75 * 2.0 ** -8
+
+
 def test_page_permutation_invariance_bitwise(ppas):
     geo = LLAMA
     shape = wl.StepShape([1, 1, 300], [2000, 77, 900])
