@@ -190,6 +190,25 @@ def test_scores_growing_along_the_context(ppas, growth):
     assert_close(host64(out), oracle_full(c), f"growth {growth}")
 
 
+def test_chunk_over_a_long_prefix(ppas):
+    """130 new tokens (two query tiles, the second ragged) over a 524,288-token
+    prefix: every (query tile, head slot) unit is cut into stream-K pieces on
+    many CTAs and merged; every element against the oracle."""
+    geo = QWEN
+    shape = wl.StepShape([130], [130 + (1 << 19)])
+    c = device_case(geo, shape, seed=45, extra_blocks=3)
+    n_kernels = ppas.ppas_attention_kernel_count(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads,
+                                                 ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens,
+                                                                                    geo.n_q_heads,
+                                                                                    geo.n_kv_heads))
+    assert n_kernels == 2  # the prefill launch and its merge
+    out = run_step(ppas, c, True)
+    torch.cuda.synchronize()
+    want = oa.paged_attention(host64(c.q), host32(c.k_cache), host32(c.v_cache), c.tables_np, shape.q_lens,
+                              shape.ctx_lens, c.scale, workers=oa.default_workers())
+    assert_close(host64(out), want, "chunk over a 512k prefix")
+
+
 def test_long_decode_rows(ppas):
     """Decode rows far longer than the workloads': 2,097,157 tokens (129
     splits of 1024 pages, merged in several rounds) against the oracle for

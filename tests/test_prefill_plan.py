@@ -85,6 +85,7 @@ def test_random_steps_plan_valid(checker):
     cases.append((16, 2, [200] * 150 + [1] * 5, [200 + 37 * i for i in range(150)] + [30000] * 5))
     cases.append((32, 8, [20000], [20500]))
     cases.append((32, 8, [65536], [66536]))
+    cases.append((16, 2, [130], [130 + (1 << 19)]))  # a chunk over a 512k-token prefix
     for case, (split, whole) in zip(cases, _run(checker, cases)):
         assert split.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {split}"
         assert whole.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {whole}"
