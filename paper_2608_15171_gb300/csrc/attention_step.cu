@@ -206,19 +206,25 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
 
     size_t u0 = 0;
     while (u0 < units.size()) {
-        // a launch takes consecutive units while its tables have room (every
-        // CTA boundary adds at most one item)
+        // a launch takes consecutive units while its tables have room (a unit
+        // is at least ceil(n_kt / kPrefillMaxPiece) items, and every CTA
+        // boundary adds at most one more)
         PrefillLaunchPlan lp;
         std::vector<int32_t> local(n_seqs, -1);
         size_t u1 = u0;
+        int64_t min_items = 0;
+        bool needs_cut = false;  // a unit longer than a piece may be
         for (; u1 < units.size(); ++u1) {
             const bool new_seq = local[units[u1].seq] < 0;
-            if (u1 - u0 + static_cast<size_t>(n_ctas) > static_cast<size_t>(kMaxPrefillWork)) break;
+            const int64_t pieces = (units[u1].n_kt + kPrefillMaxPiece - 1) / kPrefillMaxPiece;
+            if (min_items + pieces + n_ctas > kMaxPrefillWork) break;
             if (new_seq && lp.seqs.size() == static_cast<size_t>(kMaxPrefillSeqs)) break;
             if (new_seq) {
                 local[units[u1].seq] = static_cast<int32_t>(lp.seqs.size());
                 lp.seqs.push_back(units[u1].seq);
             }
+            min_items += pieces;
+            needs_cut = needs_cut || units[u1].n_kt > kPrefillMaxPiece;
         }
         int64_t total = 0, tiles = 0;
         for (size_t u = u0; u < u1; ++u) {
@@ -272,6 +278,8 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
                         int32_t take;
                         if (left <= room) {
                             take = left;
+                        } else if (room >= kPrefillMaxPiece) {
+                            take = left;  // capped below, the CTA still has room
                         } else {
                             int64_t t = std::max<int64_t>(room, 0);
                             if (left - t < kPrefillMinPiece) t = left - kPrefillMinPiece;
@@ -287,13 +295,21 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
                                 continue;
                             }
                         }
+                        // no piece longer than kPrefillMaxPiece (nor a remainder
+                        // shorter than kPrefillMinPiece after one)
+                        bool capped = false;
+                        if (take > kPrefillMaxPiece) {
+                            take = kPrefillMaxPiece;
+                            if (left - take < kPrefillMinPiece) take = left - kPrefillMinPiece;
+                            capped = true;
+                        }
                         if (out) {
                             if (static_cast<size_t>(cta) >= out->size()) out->resize(cta + 1);
                             (*out)[cta].push_back({static_cast<int32_t>(u - u0), item(un, a, a + take)});
                         }
                         load += take + kPrefillItemCost;
                         a += take;
-                        if (a < un.n_kt) {  // the unit goes on in the next CTA
+                        if (a < un.n_kt && !capped) {  // the unit goes on in the next CTA
                             ++cta;
                             load = 0;
                         }
@@ -334,7 +350,7 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
                 for (const PrefillWork &w : v) load += w.kt1 - w.kt0 + kPrefillItemCost;
                 cut_span = std::max(cut_span, load);
             }
-            if (lp.n_part == 0 || cut_span + kPrefillMergeCost >= whole_span) {
+            if (lp.n_part == 0 || (!needs_cut && cut_span + kPrefillMergeCost >= whole_span)) {
                 per_cta = std::move(whole);  // not worth the partials
                 lp.split_units.clear();
                 lp.n_part = 0;

@@ -37,6 +37,10 @@ constexpr int kMaxPrefillWork = 2400;   // items per launch (bounded by the 32 K
 constexpr int kMaxPrefillCtas = 256;    // CTAs per launch (one per SM)
 constexpr int kPrefillItemCost = 3;     // per-item overhead (Q load, pipeline fill, epilogue), in KV tiles
 constexpr int kPrefillMinPiece = 4;     // shortest piece of a split unit, in KV tiles
+// longest piece, in KV tiles: the tensor core's fp32 accumulation of O in
+// TMEM loses ~7e-7 of |O| per tile, so pieces are capped and the merge
+// (ordinary fp32) combines them
+constexpr int kPrefillMaxPiece = 512;
 constexpr int kPrefillMergeCost = 6;    // partial writes and the merge launch, in KV tiles
 constexpr uint16_t kNoPart = 0xFFFF;    // an item of an unsplit unit
 

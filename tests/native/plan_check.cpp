@@ -10,6 +10,8 @@
 //    tiles exactly once;
 //  * each piece of a split unit owns one partial slot inside the workspace,
 //    and the unit's merge entry lists exactly its pieces;
+//  * with splits allowed no item spans more than kPrefillMaxPiece KV tiles
+//    (the accumulation depth of one fp32 partial in TMEM);
 //  * without splits (a small workspace) the same coverage holds.
 // It prints one line per case: "ok <launches> <ctas> <items> <parts>
 // <max_load> <mean_load>" or "FAIL <reason>".
@@ -66,6 +68,9 @@ static std::string check(int hq, int hk, const std::vector<int32_t> &q, const st
             if (t0 >= q[s]) return "query tile";
             const int last = c[s] - q[s] + std::min(q[s], t0 + kTileQ) - 1;
             if (wk.kt0 >= wk.kt1 || wk.kt1 > last / kPrefillKT + 1) return "KV range";
+            if (split && wk.kt1 - wk.kt0 > kPrefillMaxPiece) return "piece longer than the cap";
+            if (wk.part != kNoPart && wk.kt1 - wk.kt0 < std::min(kPrefillMinPiece, last / kPrefillKT + 1))
+                return "piece shorter than the minimum";
             for (int j = wk.kt0; j < wk.kt1; ++j) {
                 const int pages = std::min(kPrefillKT / kPage, (c[s] - j * kPrefillKT + kPage - 1) / kPage);
                 if (pages < 1 || j * (kPrefillKT / kPage) + pages > (c[s] + kPage - 1) / kPage) return "page read";

@@ -70,6 +70,11 @@ def test_attention_argument_errors_before_device_work(ppas):
     with pytest.raises(E) as e:
         call(scale=-1.0)
     assert e.value.status == ppas.PPAS_ERR_INVALID_ARG
+    # a prefill row past 65535 KV tiles of 128 keys (16-bit tile indices) is refused
+    with pytest.raises(E) as e:
+        call(q_lens=[2], ctx_lens=[65535 * 128 + 1], max_blocks_per_seq=65535 * 8 + 1)
+    assert e.value.status == ppas.PPAS_ERR_UNSUPPORTED
+    assert ppas.ppas_attention_kernel_count([2], [65535 * 128], 16, 2, 0) >= 1  # the limit itself is accepted
     # a decode row longer than 2^25 tokens (2048 splits of 1024 pages) is refused
     big = (1 << 25) + 16
     with pytest.raises(E) as e:

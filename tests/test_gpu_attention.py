@@ -209,6 +209,34 @@ def test_chunk_over_a_long_prefix(ppas):
     assert_close(host64(out), want, "chunk over a 512k prefix")
 
 
+def test_chunk_at_the_longest_prefill_context(ppas):
+    """A 130-token chunk whose context ends at the longest the boundary
+    accepts for prefill rows (65535 KV tiles of 128 keys: the items' 16-bit
+    tile indices), with constant values: the output is that constant
+    whatever the weights (up to their bf16 rounding)."""
+    geo = QWEN
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    ctx = 65535 * 128
+    shape = wl.StepShape([130], [ctx])
+    nb = wl.blocks_for(ctx)
+    k_cache = torch.empty((nb, hk, 16, D), dtype=torch.bfloat16, device="cuda")
+    step = 1 << 17
+    for b0 in range(0, nb, step):
+        k_cache[b0:b0 + step] = wl.bf16_normal((min(step, nb - b0), hk, 16, D), 700 + b0 // step, "cuda")
+    v_cache = torch.full((nb, hk, 16, D), -1.25, dtype=torch.bfloat16, device="cuda")
+    tables = torch.from_numpy(wl.page_permutation(nb, 47).reshape(1, nb)).cuda()
+    q = wl.bf16_normal((130, hq, D), 48, "cuda")
+    out = torch.empty((130, hq, D), dtype=torch.float32, device="cuda")
+    ws_bytes = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, hq, hk)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ppas.ppas_attention_step(q, k_cache, v_cache, nb, tables, nb, shape.q_lens, shape.ctx_lens, hq, hk, D,
+                             geo.scale, out, True, ws, ws_bytes, err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    assert (out + 1.25).abs().max().item() <= 1.25 * 2.0 ** -8
+
+
 def test_long_decode_rows(ppas):
     """Decode rows far longer than the workloads': 2,097,157 tokens (129
     splits of 1024 pages, merged in several rounds) against the oracle for

@@ -86,6 +86,12 @@ def test_random_steps_plan_valid(checker):
     cases.append((32, 8, [20000], [20500]))
     cases.append((32, 8, [65536], [66536]))
     cases.append((16, 2, [130], [130 + (1 << 19)]))  # a chunk over a 512k-token prefix
+    # chunks at the longest context the kernel takes, and units just over,
+    # at and under the piece cap
+    cases.append((16, 2, [256], [65535 * 128]))
+    cases.append((32, 8, [128, 300], [65535 * 128 - 7, 4_000_000]))
+    for kt in (511, 512, 513, 515, 516, 1024, 1025):
+        cases.append((16, 2, [128], [kt * 128]))
     for case, (split, whole) in zip(cases, _run(checker, cases)):
         assert split.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {split}"
         assert whole.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {whole}"
