@@ -117,8 +117,12 @@ def test_kernel_count_follows_the_plan(ppas):
     assert ws > 0
     assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, ws) == 2
     assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, 0) == 1
-    # decode rows alone: one decode launch
+    # decode rows alone: one decode launch; with a chunk whose units are cut:
+    # decode, prefill and merge launches
     assert ppas.ppas_attention_kernel_count([1, 1], [3000, 5000], 16, 2, 1 << 30) == 1
+    assert ppas.ppas_attention_kernel_count([1, 1, 512], [3000, 5000, 9000], 16, 2, 1 << 30) == 3
+    # more sequences than one launch holds (whole units): two prefill launches
+    assert ppas.ppas_attention_kernel_count([200] * 150, [200 + 37 * i for i in range(150)], 16, 2, 1 << 30) == 2
     assert ppas.ppas_attention_kernel_count([], [], 16, 2, 0) == 0
     with pytest.raises(ppas.PpasError):
         ppas.ppas_attention_kernel_count([0], [5], 16, 2, 0)

@@ -209,6 +209,34 @@ def test_chunk_over_a_long_prefix(ppas):
     assert_close(host64(out), want, "chunk over a 512k prefix")
 
 
+def test_dirty_and_reused_workspace(ppas):
+    """The workspace is the caller's uninitialised memory: filled with random
+    bytes, then reused by two more steps (the split units' partials, the
+    decode partials and tickets of the step before left in it), the step
+    gives the oracle's result, bit for bit the same every time."""
+    geo = QWEN
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    shape = wl.StepShape([1, 256, 130], [20000, 40000, 9000])
+    c = device_case(geo, shape, seed=61)
+    ws_bytes = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, hq, hk)
+    # the chunks' units are cut: more workspace than the decode row's partials
+    assert ws_bytes > ppas.ppas_attention_workspace_size([1], [20000], hq, hk)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    ws = torch.randint(0, 256, (ws_bytes,), dtype=torch.uint8, device="cuda", generator=gen)
+    outs = []
+    for _ in range(3):
+        out = torch.empty((shape.total_q, hq, D), dtype=torch.float32, device="cuda")
+        err = torch.zeros(1, dtype=torch.int32, device="cuda")
+        ppas.ppas_attention_step(c.q, c.k_cache, c.v_cache, c.num_blocks, c.tables, c.width, shape.q_lens,
+                                 shape.ctx_lens, hq, hk, D, c.scale, out, True, ws, ws_bytes, err)
+        torch.cuda.synchronize()
+        assert err.item() == 0
+        outs.append(out)
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+    assert_close(host64(outs[0]), oracle_full(c), "dirty and reused workspace")
+
+
 def test_chunk_at_the_longest_prefill_context(ppas):
     """A 130-token chunk whose context ends at the longest the boundary
     accepts for prefill rows (65535 KV tiles of 128 keys: the items' 16-bit
