@@ -39,10 +39,10 @@ METRIC = "mixed prefill+decode attention step time (us) and % roofline at MBT 2k
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM traffic of one prefill-kernel launch measured by ncu, keyed by the
-# sha256 of the kernel source it was measured on (reported only while the
-# source is unchanged).
+# sha256 of the kernel's device code it was measured on (reported only while
+# that code is unchanged).
 PREFILL_TRAFFIC = {
-    "f9b1744af4d5881e": 83955200 + 21954816,   # ncu capture of one (16384, p=0) layer
+    "44b635243c3d84dc": 83955200 + 21954816,   # ncu capture of one (16384, p=0) layer
 }
 
 
@@ -56,11 +56,15 @@ def _peaks():
 
 
 def _src_hash(name):
-    """Hash of a kernel source's code: comments and blank space removed, so
-    that the ncu figures keyed by it stay valid across comment edits and go
-    null when the code changes."""
+    """Hash of a kernel source's device code: the text before its host
+    launchers (the first ``cudaError_t launch_`` definition), comments and
+    blank space removed, so that the ncu figures keyed by it stay valid across
+    comment and launcher edits and go null when the kernel's code changes."""
     with open(os.path.join(ROOT, "paper_2608_15171_gb300", "csrc", name), encoding="utf-8") as f:
         text = f.read()
+    cut = text.find("\ncudaError_t launch_")
+    if cut >= 0:
+        text = text[:cut]
     text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
     text = re.sub(r"//[^\n]*", " ", text)
     text = " ".join(text.split())

@@ -343,13 +343,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
 
 cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p,
                           cudaStream_t st) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(decode_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(kSmemBytes));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<uint64_t> smem_set{0};
+    const cudaError_t e = ensure_smem_limit(decode_attn_kernel, static_cast<int>(kSmemBytes), smem_set);
+    if (e != cudaSuccess) return e;
     if (p.n_ctas <= 0) return cudaSuccess;
     decode_attn_kernel<<<p.n_ctas, kDecodeWarps * 32, kSmemBytes, st>>>(tm_k, tm_v, p);
     return cudaGetLastError();

@@ -671,13 +671,9 @@ cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st) {
 
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
                            const PrefillParams &p, cudaStream_t st) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(kSmemBytes));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<uint64_t> smem_set{0};
+    const cudaError_t e = ensure_smem_limit(prefill_attn_kernel, static_cast<int>(kSmemBytes), smem_set);
+    if (e != cudaSuccess) return e;
     if (p.n_ctas <= 0) return cudaSuccess;
     PdlLaunch l(dim3(p.n_ctas), dim3(kThreads), kSmemBytes, st);
     return cudaLaunchKernelEx(&l.cfg, prefill_attn_kernel, tm_q, tm_k, tm_v, p);

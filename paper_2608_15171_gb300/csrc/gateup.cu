@@ -253,13 +253,9 @@ __global__ void gateup_pack_kernel(const uint4 *__restrict__ w, uint4 *__restric
 
 cudaError_t launch_gateup(const CUtensorMap &tm_x, const CUtensorMap &tm_w, const GateUpParams &p, int grid,
                           cudaStream_t st) {
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gateup_swiglu_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(kSmemG));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-    }
+    static std::atomic<uint64_t> smem_set{0};
+    const cudaError_t e = ensure_smem_limit(gateup_swiglu_kernel, static_cast<int>(kSmemG), smem_set);
+    if (e != cudaSuccess) return e;
     gateup_swiglu_kernel<<<grid, kGThreads, kSmemG, st>>>(tm_x, tm_w, p);
     return cudaGetLastError();
 }

@@ -7,6 +7,7 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <vector>
 
 #include "ppas.h"
@@ -221,6 +222,20 @@ cudaError_t launch_gateup_pack(const void *w, void *wp, int hidden, int inter, c
 // launch configuration with programmatic stream serialization: the kernel
 // may launch before its predecessor in the stream completes and orders its
 // own global accesses after it with grid_dep_wait()
+// Raises a kernel's dynamic shared memory limit, once per device (the
+// attribute belongs to the device's context); safe from several threads.
+template <typename Kernel>
+cudaError_t ensure_smem_limit(Kernel *kernel, int bytes, std::atomic<uint64_t> &done) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = dev >= 0 && dev < 64 ? uint64_t{1} << dev : 0;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+    return e;
+}
+
 struct PdlLaunch {
     cudaLaunchAttribute attr[1];
     cudaLaunchConfig_t cfg;
