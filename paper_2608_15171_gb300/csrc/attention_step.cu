@@ -61,11 +61,17 @@ SideStream *side_stream() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
     SideStream &ss = g_side[dev];
-    if (!ss.stream) {
-        if (cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
-        if (cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming) != cudaSuccess ||
-            cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming) != cudaSuccess)
-            return nullptr;
+    if (!ss.stream && cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking) != cudaSuccess) {
+        ss.stream = nullptr;
+        return nullptr;
+    }
+    if (!ss.fork && cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming) != cudaSuccess) {
+        ss.fork = nullptr;
+        return nullptr;
+    }
+    if (!ss.join && cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming) != cudaSuccess) {
+        ss.join = nullptr;
+        return nullptr;
     }
     return &ss;
 }
@@ -621,10 +627,11 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
 
     // with prefill chunks in the same step the decode launch is forked onto
     // a side stream after the prefill launch and joined back
-    SideStream *side = dp.rows.empty() ? nullptr : side_stream();
+    // (the side stream and its events are created, and used, under the lock)
     std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
+    if (!dp.rows.empty()) side_lock.lock();
+    SideStream *side = dp.rows.empty() ? nullptr : side_stream();
     if (side) {
-        side_lock.lock();
         if (cudaEventRecord(side->fork, cs) != cudaSuccess ||
             cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
             return PPAS_ERR_CUDA;
