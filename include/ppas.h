@@ -4,10 +4,12 @@
  *
  * The library is a plain shared object (libppas.so).  Every entry point takes
  * plain host or device pointers and sizes; nothing here mentions a framework
- * type.  The library keeps no global state apart from a per-device cache of
- * driver entry points and the fixed scratch array of
- * ppas_attention_step_noalloc; the only stateful object is the opaque
- * planner ppas_sched, which owns the free list of KV blocks.
+ * type.  The library keeps no global state apart from per-device caches
+ * (driver entry points, the SM count, the kernels' shared-memory limits, one
+ * side stream with two events, all created on first use and thread-safe)
+ * and the fixed scratch array of ppas_attention_step_noalloc; the only
+ * stateful object is the opaque planner ppas_sched, which owns the free list
+ * of KV blocks.
  *
  * Ownership: the caller owns every buffer passed in (inputs, caches,
  * outputs, workspace, error flag, plan arrays).  No call allocates device
