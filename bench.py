@@ -37,6 +37,7 @@ from paper_2608_15171_gb300 import workloads as wl  # noqa: E402
 
 METRIC = "mixed prefill+decode attention step time (us) and % roofline at MBT 2k/16k"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+NOMINAL_HBM_GBS = 7900.0   # GB300 HBM3e, nominal
 
 # DRAM traffic of one prefill-kernel launch measured by ncu, keyed by the
 # sha256 of the kernel's device code it was measured on (reported only while
@@ -395,6 +396,32 @@ def _llama_bench(torch, ppas, dist, dev, stream, peaks, steps, warmup, rank):
             "peak_kind": "measured burst bf16 and HBM copy", **res}
 
 
+def _decode_bench(torch, ppas, dist, dev, stream, peaks, steps, warmup, rank):
+    """The split-K decode kernel alone: the 16 decode rows of the Llama-3.1-8B
+    MBT 2k step (contexts ~U[30000, 30064), 32q/8kv/d128; K and V of every
+    context token once per kv-head, ~1.97 GB a layer), attention calls only,
+    32 layers over 4 buffer sets, each far larger than L2.  HBM-bound, so it
+    is reported against the measured copy bandwidth and the nominal 7.9 TB/s."""
+    geo = wl.LLAMA31_8B
+    full = wl.llama_lo_step(0)
+    rows = [i for i, q in enumerate(full.q_lens) if q == 1]
+    shape = wl.StepShape([1] * len(rows), [full.ctx_lens[i] for i in rows])
+    W = _setup_step(torch, ppas, geo, shape, dev, seed=5, n_sets=4)
+    ms, _, _, _ = _timed(torch, dist, lambda tm: _high_step(torch, ppas, W, stream, append=False), steps, warmup,
+                         stream, rank, False)
+    assert W.err.item() == 0, f"device error flag {W.err.item()}"
+    us = ms * 1e3 / steps / geo.n_layers
+    gbs = wl.step_bytes(shape, geo) / (us * 1e-6) / 1e9
+    del W
+    torch.cuda.empty_cache()
+    return {"workload": f"{len(rows)} decode rows of the Llama-3.1-8B MBT 2048 step alone (ctx ~U[30000,30064)), "
+                        "attention calls only, 32 layers",
+            "kernel": "decode_attn_kernel", "us_per_layer": round(us, 1),
+            "bytes_per_layer": wl.step_bytes(shape, geo), "hbm_gbs": round(gbs, 1),
+            "frac_vs_measured_hbm": round(gbs / peaks["hbm_gbs"], 4),
+            "frac_vs_nominal_hbm": round(gbs / NOMINAL_HBM_GBS, 4)}
+
+
 def _burst_replay(torch, ppas, geo, dev, peaks, rates=(0.5, 1.0, 2.0, 4.0), seed=0):
     """The burst replay workload: a Poisson burst of 16 requests (prompts
     ~U[20000, 30000], outputs ~U[16, 64]) at each rate, planned by the P-PAS
@@ -547,6 +574,7 @@ def run_ours(args, rank, world, dist):
     mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
     gateup = _gateup_bench(torch, ppas, dev, stream, peaks)
     llama = _llama_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
+    decode = _decode_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     burst = _burst_replay(torch, ppas, geo, dev, peaks)
 
     line = {
@@ -576,6 +604,7 @@ def run_ours(args, rank, world, dist):
         "mbt_sweep": mbt_sweep,
         "gateup": gateup,
         "llama": llama,
+        "decode": decode,
         "burst_replay": burst,
         "e2e": e2e,
         "gpu_launches": launches // args.steps * args.steps,
