@@ -334,6 +334,45 @@ def _mbt_sweep(torch, ppas, geo, dev, stream, reps=10, warmup=3, n_sets=8):
             "ratio_to_16k": {k: round(v / res["16384"], 3) for k, v in res.items()}}
 
 
+def _append_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3, n_layers=36):
+    """The KV append alone: the 16,384 new tokens of the (16384, p=0) chunk
+    (Qwen2.5-3B geometry, 2 kv-heads) written into 36 distinct layers' paged
+    caches in random block order, back to back; the median over repeats of
+    the 36 launches.  Algorithmic bytes per launch: the new K and V read, the
+    same bytes written into the cache pages, the slot ids read."""
+    geo = wl.QWEN25_3B
+    T, hk, D = 16384, geo.n_kv_heads, geo.head_dim
+    nb = wl.blocks_for(T) + 13
+    perm = np.asarray(wl.page_permutation(nb, 11), dtype=np.int64)
+    t = np.arange(T)
+    slots = torch.from_numpy((perm[t // 16] * 16 + t % 16).astype(np.int32)).to(dev)
+    layers = [(wl.bf16_normal((T, hk, D), 600 + i, dev), wl.bf16_normal((T, hk, D), 700 + i, dev),
+               torch.zeros((nb, hk, 16, D), dtype=torch.bfloat16, device=dev),
+               torch.zeros((nb, hk, 16, D), dtype=torch.bfloat16, device=dev)) for i in range(n_layers)]
+    err = torch.zeros(1, dtype=torch.int32, device=dev)
+    times = []
+    for r in range(warmup + reps):
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for kn, vn, kc, vc in layers:
+            ppas.ppas_kv_append(kn, vn, slots, T, kc, vc, nb, hk, D, err, stream)
+        e1.record(stream)
+        times.append((e0, e1))
+    torch.cuda.synchronize()
+    assert err.item() == 0, f"device error flag {err.item()}"
+    ts = sorted(a.elapsed_time(b) for a, b in times[warmup:])
+    us = ts[len(ts) // 2] * 1e3 / n_layers
+    by = 2 * (T * hk * D * 2 * 2) + T * 4
+    gbs = by / (us * 1e-6) / 1e9
+    del layers
+    torch.cuda.empty_cache()
+    return {"workload": "KV append of 16,384 tokens (2 kv-heads, d 128, bf16) into 36 layers' paged caches, "
+                        "random block order", "kernel": "kv_append_kernel", "us_per_launch": round(us, 2),
+            "bytes_per_launch": by, "hbm_gbs": round(gbs, 1),
+            "frac_vs_measured_hbm": round(gbs / peaks["hbm_gbs"], 4)}
+
+
 def _gateup_bench(torch, ppas, dev, stream, peaks, reps=10, warmup=3):
     """The gate-up projection with the fused gated activation for a
     16,384-token prompt of the Qwen2.5-3B MLP (hidden 2048, intermediate
@@ -573,6 +612,7 @@ def run_ours(args, rank, world, dist):
     del H
     mbt_sweep = _mbt_sweep(torch, ppas, geo, dev, stream)
     gateup = _gateup_bench(torch, ppas, dev, stream, peaks)
+    append = _append_bench(torch, ppas, dev, stream, peaks)
     llama = _llama_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     decode = _decode_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     burst = _burst_replay(torch, ppas, geo, dev, peaks)
@@ -603,6 +643,7 @@ def run_ours(args, rank, world, dist):
         "mbt2k": mbt2k,
         "mbt_sweep": mbt_sweep,
         "gateup": gateup,
+        "append": append,
         "llama": llama,
         "decode": decode,
         "burst_replay": burst,
