@@ -74,3 +74,27 @@ def test_reference_arm_nonzero_rank_does_no_work():
         steps, warmup, cpu_seconds = 1, 0, 0.1
 
     assert bench.run_reference(Args(), 1, 2) is None
+
+
+def test_traffic_key_follows_the_device_code(tmp_path, monkeypatch):
+    """The ncu traffic in the bench line is keyed by a hash of the prefill
+    kernel's device code: comment and host-launcher edits keep the key, an
+    edit of the kernel's code changes it (and the bench then reports null)."""
+    sys.path.insert(0, ROOT)
+    import bench
+    src = os.path.join(ROOT, "paper_2608_15171_gb300", "csrc", "attn_prefill.cu")
+    text = open(src, encoding="utf-8").read()
+    assert bench.PREFILL_TRAFFIC.get(bench._src_hash("attn_prefill.cu")) is not None
+    csrc = tmp_path / "paper_2608_15171_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+
+    def key(t):
+        (csrc / "attn_prefill.cu").write_text(t, encoding="utf-8")
+        return bench._src_hash("attn_prefill.cu")
+
+    base = key(text)
+    cut = text.index("\ncudaError_t launch_")
+    assert key(text.replace("// ", "//  note: ", 1)) == base
+    assert key(text[:cut] + "\n// a launcher comment" + text[cut:].replace("return", "return ", 1)) == base
+    assert key(text[:cut].replace("kNK = 3", "kNK = 2", 1) + text[cut:]) != base
