@@ -38,6 +38,11 @@ from paper_2608_15171_gb300 import workloads as wl  # noqa: E402
 METRIC = "mixed prefill+decode attention step time (us) and % roofline at MBT 2k/16k"
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 NOMINAL_HBM_GBS = 7900.0   # GB300 HBM3e, nominal
+# the workload both arms report (the GPU arm times it; the reference arm
+# extrapolates the oracle's time on a sample of it)
+HEADLINE_WORKLOAD = ("MBT 16384 low pressure: 25,000-token prompt planned into chunks (16384, p=0) and "
+                     "(8616, p=16384); Qwen2.5-3B attention geometry 16q/2kv/d128, 36 layers; "
+                     "plan + kv append + attention per layer")
 
 # DRAM traffic of one prefill-kernel launch measured by ncu, keyed by the
 # sha256 of the kernel's device code it was measured on (reported only while
@@ -426,7 +431,7 @@ def _llama_bench(torch, ppas, dist, dev, stream, peaks, steps, warmup, rank):
         step_us = ms * 1e3 / steps
         roof = _roofline_time_us(W.shape, geo, peaks, False) * geo.n_layers
         roof_sus = _roofline_time_us(W.shape, geo, peaks, True) * geo.n_layers
-        res[name] = {"q_lens": W.shape.q_lens, "ctx_lens": W.shape.ctx_lens, "step_us": round(step_us, 1),
+        res[name] = {"step_us": round(step_us, 1),
                      "us_per_layer": round(step_us / geo.n_layers, 1), "roofline_us": round(roof, 1),
                      "frac": round(roof / step_us, 4), "frac_vs_sustained_peak": round(roof_sus / step_us, 4)}
         del W
@@ -488,6 +493,31 @@ def _burst_replay(torch, ppas, geo, dev, peaks, rates=(0.5, 1.0, 2.0, 4.0), seed
     return {"workload": "Poisson burst of 16 requests, prompts ~U[20000,30000], outputs ~U[16,64], P-PAS threshold 2, "
                         "MBT 16384/2048, every iteration on 36 layers (append + attention), closed loop",
             "unit": "us", "rates_req_per_s": res}
+
+
+def _policy_compare(geo, dev, rates=(0.4, 1.0), seed=0, time_scale=40.0):
+    """Closed-loop comparison of P-PAS with the static budgets MBT 2k and MBT
+    16k (Sections 4.1, 4.4 and 5.1), reduced to fit the bench: the 50 s
+    alternating steady/burst trace at two burst rates (the rates of the
+    paper's A100 runs) and one seed, every time compressed x40 (phases
+    0.25 s, rates x40: the same requests in the same order), each iteration
+    executed on all 36 layers (appends + attention only; no projections,
+    MLP or sampling) with its measured time driving the clock.  Per policy
+    and rate: average and P95 latency, TTFT, TPOT, makespan (seconds of the
+    compressed trace); I_m of P-PAS over each baseline across the rates."""
+    from paper_2608_15171_gb300 import serving
+    import torch
+    pols = ("P-PAS", "MBT 2k", "MBT 16k")
+    res = serving.sweep(list(rates), [seed], time_scale, pols, geo=geo, device=dev, log=lambda *_: None)
+    torch.cuda.empty_cache()
+    keys = ("avg_latency_s", "p95_latency_s", "avg_ttft_s", "avg_tpot_s", "makespan_s")
+    per = {p: {str(r): {k: round(res[p][r][k], 4) for k in keys} for r in rates} for p in pols}
+    imp = {b: {k: round(serving.improvement([res["P-PAS"][r][k] for r in rates], [res[b][r][k] for r in rates]), 2)
+               for k in keys} for b in pols if b != "P-PAS"}
+    return {"workload": f"50 s alternating trace (steady 0.2 req/s, bursts at {list(rates)} req/s, 10 s phases), "
+                        f"25k prompts, 32 outputs, seed {seed}, times compressed x{time_scale:g}; attention only "
+                        f"(append + attention, 36 layers per iteration)",
+            "per_policy": per, "improvement_pct": imp}
 
 
 def _roofline_time_us(shape, geo, peaks, sustained):
@@ -560,7 +590,7 @@ def run_ours(args, rank, world, dist):
     avg_launch_ms = sum(first) / len(first)
     attn_flops_per_launch = wl.step_flops(shapes[0], geo)
     achieved = attn_flops_per_launch / (avg_launch_ms * 1e-3) / 1e12
-    peak = peaks["bf16_tflops_sustained"]
+    peak = peaks["bf16_tflops"]
     # the step roofline of the metric: max(FLOPs / burst bf16 peak, bytes / HBM)
     roof_step_us = sum(_roofline_time_us(sh, geo, peaks, False) for sh in shapes) * geo.n_layers
     roof_step_sus_us = sum(_roofline_time_us(sh, geo, peaks, True) for sh in shapes) * geo.n_layers
@@ -584,8 +614,8 @@ def run_ours(args, rank, world, dist):
                      "output out on another, overlapping the other layers' compute; both joined before the "
                      "step's end event"}
     del host
-    cpu_w = {"k": W.k_cache[0], "v": W.v_cache[0]}
-    W_low = W
+    del W
+    torch.cuda.empty_cache()
 
     # ---- high pressure (MBT 2k with 8 decodes)
     H = _setup_high(torch, ppas, geo, dev)
@@ -601,7 +631,6 @@ def run_ours(args, rank, world, dist):
     attn_h_ms = ms_ha / args.steps
     mbt2k = {
         "workload": "MBT 2048: 4x512 chunks, prefixes ~U[0,24576) + 8 decodes ctx ~U[25000,25032), 36 layers",
-        "q_lens": H.shape.q_lens, "ctx_lens": H.shape.ctx_lens,
         "step_us": round(hs_us, 1), "attention_us_per_layer": round(attn_h_ms * 1e3 / geo.n_layers, 2),
         "roofline_us": round(roof_h_us, 1), "peak_kind": f"{peaks_kind} burst bf16 and HBM copy",
         "frac": round(roof_h_us / hs_us, 4),
@@ -616,21 +645,22 @@ def run_ours(args, rank, world, dist):
     llama = _llama_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     decode = _decode_bench(torch, ppas, dist, dev, stream, peaks, args.steps, args.warmup, rank)
     burst = _burst_replay(torch, ppas, geo, dev, peaks)
+    policy = _policy_compare(geo, dev) if not args.no_policy else None
 
     line = {
         "metric": METRIC, "value": round(step_us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": False,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "MBT 16384 low pressure: 25,000-token prompt planned into chunks (16384, p=0) and "
-                               "(8616, p=16384); Qwen2.5-3B attention geometry 16q/2kv/d128, 36 layers; "
-                               "plan + kv append + attention per layer",
+        "config": {"workload": HEADLINE_WORKLOAD,
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (distinct buffers per layer)",
                    "step": "2 scheduler iterations x 36 layers"},
         "roofline": {"bound": "tensor", "kernel": "prefill_attn_kernel",
                      "launch": "one (16384, p=0) layer: 16384 queries x 16 heads over their causal prefix",
                      "achieved": round(achieved, 1),
                      "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-                     "peak_kind": f"{peaks_kind} sustained bf16", "traffic": traffic,
+                     "peak_kind": f"{peaks_kind} burst bf16",
+                     "frac_vs_sustained_peak": round(achieved / peaks["bf16_tflops_sustained"], 4),
+                     "traffic": traffic,
                      "avg_launch_us": round(avg_launch_ms * 1e3, 1),
                      "flops_per_launch": attn_flops_per_launch},
         "step_roofline": {"roofline_us": round(roof_step_us, 1), "peak_kind": f"{peaks_kind} burst bf16 and HBM copy",
@@ -647,58 +677,149 @@ def run_ours(args, rank, world, dist):
         "llama": llama,
         "decode": decode,
         "burst_replay": burst,
-        "e2e": e2e,
-        "gpu_launches": launches // args.steps * args.steps,
-        "clocks": clocks,
+        "policy_comparison": policy,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(W_low, cpu_w, torch, args)
+        line["cpu_baseline"] = cpu_baseline(torch, args, dev)
+    line["e2e"] = e2e
+    line["gpu_launches"] = launches // args.steps * args.steps
+    line["clocks"] = clocks
+    # the step-roofline fraction of every configuration, last in the line
+    # so that a record keeping only the line's tail still holds them
+    line["targets"] = {
+        "peak": f"{peaks_kind} burst {peaks['bf16_tflops']} TF/s, HBM {peaks['hbm_gbs']} GB/s",
+        "mbt16k": {"frac": line["step_roofline"]["frac"], "target": 0.60, "step_us": line["value"]},
+        "mbt2k": {"frac": mbt2k["frac"], "target": 0.50, "us_per_layer": round(mbt2k["step_us"] / 36, 1)},
+        "llama16k": {"frac": llama["mbt16k"]["frac"], "target": 0.60, "us_per_layer": llama["mbt16k"]["us_per_layer"]},
+        "llama2k": {"frac": llama["mbt2k"]["frac"], "target": 0.50, "us_per_layer": llama["mbt2k"]["us_per_layer"]},
+        "prefill_kernel": {"tflops": round(achieved, 1), "frac": round(achieved / peak, 4)},
+        "decode_kernel": {"gbs": decode["hbm_gbs"], "frac": decode["frac_vs_measured_hbm"]},
+        "replay_frac": {r: {k[2:]: v["frac"] for k, v in d.items() if k.startswith("B=")}
+                        for r, d in burst["rates_req_per_s"].items()},
+    }
+    if policy is not None:
+        line["targets"]["policy_I_avg_latency_pct"] = {
+            b: round(v["avg_latency_s"], 2) for b, v in policy["improvement_pct"].items()}
     return line
 
 
-def _oracle_sample(kc, vc, table, geo, rows, workers):
-    """Oracle on the last ``rows`` query tokens of the first 16384-token chunk
-    (all 16 heads); returns (seconds, causal pairs per head)."""
+def _blas_threads():
+    """Threads of the BLAS numpy uses in each oracle call: threadpoolctl when
+    it is installed, else the library's own thread count read through its
+    exported getter, else the environment's setting (None if none of these
+    says)."""
+    np.dot(np.ones((64, 64)), np.ones((64, 64)))  # make sure the BLAS is loaded
+    try:
+        import threadpoolctl
+        info = [d for d in threadpoolctl.threadpool_info() if d.get("user_api") == "blas"]
+        if info:
+            return int(info[0]["num_threads"])
+    except Exception:
+        pass
+    try:
+        import ctypes
+        with open("/proc/self/maps") as f:
+            libs = sorted({ln.split()[-1] for ln in f if "openblas" in ln.lower() and ".so" in ln})
+        for path in libs:
+            lib = ctypes.CDLL(path)
+            for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_",
+                        "openblas_get_num_threads"):
+                fn = getattr(lib, sym, None)
+                if fn is not None:
+                    fn.restype = ctypes.c_int
+                    return int(fn())
+    except Exception:
+        pass
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    return None
+
+
+def _oracle_layer(torch, geo, shape, seed, workers, sample_rows=None, device="cpu"):
+    """Times the float64 oracle on one layer of a step: seeded N(0,1) bf16 Q
+    and K/V caches (every context filled, pages in a seeded random order),
+    then ``oracle.attention.paged_attention`` over all rows, or with
+    ``sample_rows`` over the last ``sample_rows`` query tokens of every
+    prefill chunk (their whole causal context, all heads) plus the first two
+    decode rows.  Returns (seconds, causal (query, key) pairs per q-head computed)."""
     from oracle import attention as oa
-    L = 16384
-    q = wl.bf16_normal((rows, geo.n_q_heads, geo.head_dim), 77, "cpu").to(torch_float64())
+    need = sum(wl.blocks_for(c) for c in shape.ctx_lens)
+    nb = need + 5
+    tables = wl.literal_tables(shape, wl.page_permutation(nb, seed))
+    hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
+    kc = wl.bf16_normal((nb, hk, 16, D), seed * 7 + 1, device).float().cpu().numpy()
+    vc = wl.bf16_normal((nb, hk, 16, D), seed * 7 + 2, device).float().cpu().numpy()
+    run = shape
+    if sample_rows is not None:
+        # the last sample_rows tokens of every chunk, the first 2 decode rows
+        dec = [i for i, q in enumerate(shape.q_lens) if q == 1][:2]
+        keep = dec + [i for i, q in enumerate(shape.q_lens) if q > 1]
+        run = wl.StepShape([min(shape.q_lens[i], sample_rows) for i in keep], [shape.ctx_lens[i] for i in keep])
+        tables = tables[keep]
+    q = wl.bf16_normal((run.total_q, hq, D), seed * 7 + 3, device).double().cpu().numpy()
     t0 = time.perf_counter()
-    oa.paged_attention(q.numpy(), kc, vc, table, [rows], [L], geo.scale, workers=workers)
-    dt = time.perf_counter() - t0
-    p = L - rows
-    return dt, rows * p + rows * (rows + 1) // 2
+    oa.paged_attention(q, kc, vc, tables, run.q_lens, run.ctx_lens, geo.scale, workers=workers)
+    return time.perf_counter() - t0, wl.step_pairs(run)
 
 
-def torch_float64():
-    import torch
-    return torch.float64
+# the oracle's per-config timing, cheapest first: (name, geometry, steps of
+# one layer, layers per step, what one bench step of that config is)
+def _cpu_configs():
+    return [("1 tiny", wl.QWEN25_3B, wl.tiny_steps(), 1, "the 4 steps of one layer"),
+            ("3 MBT 2k", wl.QWEN25_3B, [wl.high_pressure_step(0)], 36, "one step x 36 layers"),
+            ("2 MBT 16k", wl.QWEN25_3B, wl.low_pressure_steps(), 36, "2 iterations x 36 layers"),
+            ("5-lo Llama MBT 2k", wl.LLAMA31_8B, [wl.llama_lo_step(0)], 32, "one step x 32 layers"),
+            ("5-hi Llama MBT 16k", wl.LLAMA31_8B, [wl.llama_hi_step(0)], 32, "one step x 32 layers")]
 
 
-def _workload_pairs(geo):
-    return sum(wl.step_pairs(sh) for sh in wl.low_pressure_steps()) * geo.n_layers
-
-
-def cpu_baseline(W, cache, torch, args):
+def cpu_baseline(torch, args, device="cpu"):
+    """The float64 oracle as it stands, on this host's cores: for every
+    config with an attention step, one full layer timed (all rows, all
+    heads) and extrapolated to the config's layers, cheapest config first;
+    a config whose full layer would not fit the remaining time budget
+    (estimated from the rate measured so far) is timed on a sample instead
+    (the last 256 query tokens of every chunk plus two decode rows) and
+    extrapolated by causal pair count; once the budget is spent the rest
+    are skipped.  ``value`` is the headline
+    workload's (MBT 16k, 2 iterations x 36 layers)."""
     from oracle import attention as oa
-    geo = W.geo
-    kc = cache["k"].float().cpu().numpy()
-    vc = cache["v"].float().cpu().numpy()
-    table = np.array([W.perm[: wl.blocks_for(W.prompt)]], dtype=np.int64)
     workers = oa.default_workers()
-    budget_s = args.cpu_seconds
-    total_t, total_pairs, n = 0.0, 0, 0
-    rows = 256
-    while total_t < budget_s and n < 64:
-        dt, pairs = _oracle_sample(kc, vc, table, geo, rows, workers)
-        total_t += dt
-        total_pairs += pairs
-        n += 1
-    us_per_step = total_t / total_pairs * _workload_pairs(geo) * 1e6
-    return {"value": round(us_per_step, 1), "unit": "us", "cores": workers, "kind": "oracle",
-            "sample": f"{n} runs of the oracle on the last {rows} query tokens (all 16 heads) of the "
-                      f"16384-token chunk over its full 16384-token context, {total_t:.1f} s, "
-                      f"extrapolated by causal pair count to the whole step (2 iterations x 36 layers)",
-            "planner": _planner_timing()}
+    blas = _blas_threads()
+    budget = float(args.cpu_seconds)
+    spent, rate = 0.0, None          # rate: pair-heads per second
+    per = {}
+    for name, geo, steps, layers, what in _cpu_configs():
+        work = sum(wl.step_pairs(s) for s in steps) * geo.n_q_heads
+        if spent >= budget:
+            per[name] = {"kind": "skipped: time budget spent", "step": what, "geometry": geo.name}
+            continue
+        full = rate is None or work / rate <= budget - spent
+        secs, done = 0.0, 0
+        for i, sh in enumerate(steps):
+            dt, pairs = _oracle_layer(torch, geo, sh, 11 + i, workers, None if full else 256, device)
+            secs += dt
+            done += pairs * geo.n_q_heads
+        spent += secs
+        if full:
+            rate = done / secs if rate is None else max(rate, done / secs)
+        us_layer = secs / done * work * 1e6          # one layer of every step
+        per[name] = {"kind": "full layer" if full else "sample: last 256 tokens of each chunk + 2 decode rows",
+                     "seconds": round(secs, 2), "us_per_step": round(us_layer * layers, 1),
+                     "extrapolated": f"x{layers} layers" if layers > 1 else None,
+                     "step": what, "geometry": geo.name}
+        if not full:
+            per[name]["extrapolated"] = f"x{work / done:.4g} by causal pairs" + (
+                f", x{layers} layers" if layers > 1 else "")
+    head = per["2 MBT 16k"]
+    if "us_per_step" not in head:
+        return {"value": None, "unit": "us", "cores": workers, "blas_threads": blas, "kind": "oracle",
+                "sample": "time budget spent before the headline workload", "per_config": per}
+    return {"value": head["us_per_step"], "unit": "us", "cores": workers, "blas_threads": blas,
+            "kind": "oracle", "extrapolated": True,
+            "sample": f"headline = config 2 ({head['kind']}, {head['seconds']} s) {head['extrapolated']}; "
+                      f"oracle = float64 numpy, thread pool of {workers}, budget {budget:.0f} s",
+            "per_config": per}
 
 
 def _planner_timing():
@@ -723,37 +844,45 @@ def _planner_timing():
 
 
 def run_reference(args, rank, world):
-    """The float64 oracle as the reference arm, on this host's cores."""
+    """The float64 oracle as the reference arm, on this host's cores: each
+    step runs the oracle on a bounded sample of the headline workload (the
+    last 128 query tokens of both chunks, all heads, over their full causal
+    context) and is extrapolated by causal pair count to the whole step."""
     if rank != 0:
         return None
     from oracle import attention as oa
+    import torch
     geo = wl.QWEN25_3B
-    L = 16384
-    nb = wl.blocks_for(L)
-    perm = wl.page_permutation(nb, 0)
-    table = np.array([perm], dtype=np.int64)
-    kc = wl.bf16_normal((nb, geo.n_kv_heads, 16, geo.head_dim), 1, "cpu").float().numpy()
-    vc = wl.bf16_normal((nb, geo.n_kv_heads, 16, geo.head_dim), 2, "cpu").float().numpy()
     workers = oa.default_workers()
     rows = 128
+    steps = wl.low_pressure_steps()
+    full_pairs = sum(wl.step_pairs(sh) for sh in steps) * geo.n_layers
+
+    def one():
+        t, p = 0.0, 0
+        for i, sh in enumerate(steps):
+            dt, pairs = _oracle_layer(torch, geo, sh, 11 + i, workers, rows)
+            t += dt
+            p += pairs
+        return t, p
+
     for _ in range(args.warmup):
-        _oracle_sample(kc, vc, table, geo, rows, workers)
+        one()
     total_t, total_pairs = 0.0, 0
     for _ in range(args.steps):
-        dt, pairs = _oracle_sample(kc, vc, table, geo, rows, workers)
+        dt, pairs = one()
         total_t += dt
         total_pairs += pairs
-    us = total_t / total_pairs * _workload_pairs(geo) * 1e6
-    sample = (f"each step: the oracle on the last {rows} query tokens (16 heads) of the 16384-token chunk over its "
-              f"full context; extrapolated by causal pair count to the whole step (2 iterations x 36 layers)")
+    us = total_t / total_pairs * full_pairs * 1e6
+    sample = (f"each step: the oracle on the last {rows} query tokens (16 heads) of both chunks over their full "
+              f"causal context; extrapolated by causal pair count (x{full_pairs * args.steps / total_pairs:.4g}) "
+              f"to the whole step (2 iterations x 36 layers)")
     return {"metric": METRIC, "value": round(us, 1), "unit": "us", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(us / 1e3, 3), "higher_is_better": False, "scaling": "weak",
-            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": "MBT 16384 low pressure: 25,000-token prompt as chunks (16384, p=0) and "
-                                   "(8616, p=16384); Qwen2.5-3B attention geometry, 36 layers",
-                       "parallelism": "cpu oracle"},
-            "cpu_baseline": {"value": round(us, 1), "unit": "us", "cores": workers, "kind": "oracle",
-                             "sample": sample},
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference", "extrapolated": True,
+            "config": {"workload": HEADLINE_WORKLOAD, "parallelism": "cpu oracle"},
+            "cpu_baseline": {"value": round(us, 1), "unit": "us", "cores": workers, "blas_threads": _blas_threads(),
+                             "kind": "oracle", "extrapolated": True, "sample": sample},
             "e2e": {"value": round(us, 1), "unit": "us", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -764,7 +893,9 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-policy", action="store_true", help="skip the closed-loop policy comparison")
+    ap.add_argument("--cpu-seconds", type=float, default=60.0,
+                    help="time budget of the oracle's per-config timing (full layers while they fit)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -254,22 +254,32 @@ ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int
  * program whose device memory belongs to another allocator).
  *
  * Same arguments, layouts and results as ppas_attention_step, minus the
- * workspace: the split-K decode scratch lives in a fixed array of
- * PPAS_NOALLOC_SCRATCH_BYTES inside the library's device memory, which every
- * GPU that loads the library holds until the process exits.  The call makes
- * no cudaMalloc, cudaFree or other allocating call.
- *  - A step whose scratch (ppas_attention_workspace_size) exceeds
- *    PPAS_NOALLOC_SCRATCH_BYTES is rejected with PPAS_ERR_CAPACITY before any
- *    device work.
- *  - The first call on a device (with scratch to use) looks up the array's
- *    device address with that device current; make that first call before
- *    any stream capture.  PPAS_ERR_CUDA if the lookup fails.
+ * workspace: the scratch lives in a fixed array of
+ * PPAS_NOALLOC_SCRATCH_BYTES (64 MiB) inside the library's device memory,
+ * which every GPU that loads the library holds until the process exits.
+ * The call makes no cudaMalloc, cudaFree or other allocating call.
+ *  - The split-K decode scratch of the step must fit the array, else the
+ *    step is rejected with PPAS_ERR_CAPACITY before any device work.
+ *  - When the prefill tiles' split partials also fit beside it
+ *    (ppas_attention_workspace_size <= PPAS_NOALLOC_SCRATCH_BYTES, true for
+ *    every workload of the paper's configurations) the step runs exactly as
+ *    ppas_attention_step with a full workspace.  Otherwise the prefill
+ *    tiles run unsplit: same results up to rounding, except that a query
+ *    tile over a context longer than 65,536 keys then accumulates in one
+ *    piece, whose fp32 tensor-core accumulation drifts towards smaller
+ *    magnitude (~4e-4 relative at 110k keys, ~5e-3 at 880k).
+ *  - The first call on a device (with rows to run) does the library's
+ *    one-time set-up for that device with it current: it looks up the
+ *    array's device address, sets the kernels' shared-memory limits and
+ *    creates the side stream and two events of mixed steps.  Make that first
+ *    call before any stream capture and before a phase in which nothing may
+ *    be created.  PPAS_ERR_CUDA if the set-up fails.
  *  - All calls share one array, which keeps the last call's contents (the
  *    parts that must start at zero are cleared on the stream by every call).
  *    Calls whose work overlaps on the GPU (other streams, other host threads)
  *    race on it: serialise them.
  * ------------------------------------------------------------------------- */
-#define PPAS_NOALLOC_SCRATCH_BYTES (4 * 1024 * 1024)
+#define PPAS_NOALLOC_SCRATCH_BYTES (64 * 1024 * 1024)
 
 ppas_status ppas_attention_step_noalloc(const void *q, const void *k_cache, const void *v_cache,
                                         int32_t num_blocks, const int32_t *d_block_tables,

@@ -6,15 +6,19 @@
 // must not allocate afterwards (cudaMalloc can synchronise the device, stall
 // the loop or fail under memory pressure), or a host program whose memory is
 // owned by someone else's allocator and that only passes in the tensors it
-// was given.  For them this file keeps the split-K decode scratch in a
-// fixed-size array in the library's own device memory, so a call needs only
-// the inputs and outputs.
+// was given.  For them this file keeps the step's scratch (the decode
+// splits' partials and, when they fit beside them, the prefill pieces'
+// partials) in a fixed-size array in the library's own device memory, so a
+// call needs only the inputs and outputs.
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds it (PPAS_NOALLOC_SCRATCH_BYTES) until the process exits.
 // Host code may not use the array's name as a device address, so the first
 // call on each device looks the address up with cudaGetSymbolAddress while
-// that device is current, and later calls reuse it.
+// that device is current, and later calls reuse it.  That first call also
+// does the library's other one-time set-up for the device (the kernels'
+// shared-memory limits, the side stream and events of mixed steps), so that
+// no later call creates anything.
 #include <mutex>
 
 #include "ppas_internal.h"
@@ -36,6 +40,7 @@ void *scratch_on_current_device() {
     if (!g_scratch_ptr[dev]) {
         void *ptr = nullptr;
         if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return nullptr;
+        if (ppas::prepare_current_device() != cudaSuccess) return nullptr;
         g_scratch_ptr[dev] = ptr;
     }
     return g_scratch_ptr[dev];
@@ -49,8 +54,9 @@ extern "C" ppas_status ppas_attention_step_noalloc(const void *q, const void *k_
                                                    const int32_t *h_ctx_lens, int32_t n_seqs, int32_t n_q_heads,
                                                    int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
                                                    int32_t out_is_fp32, int32_t *d_err_flag, void *stream) {
-    // the scratch this step needs must fit the fixed array (checked before any
-    // CUDA call); prefill tiles run unsplit when their split partials do not fit
+    // the decode scratch this step needs must fit the fixed array (checked
+    // before any CUDA call); the prefill tiles' split partials are used when
+    // they fit beside it, else the prefill tiles run unsplit
     const size_t need = ppas::workspace_min_size(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
     if (need > static_cast<size_t>(PPAS_NOALLOC_SCRATCH_BYTES)) return PPAS_ERR_CAPACITY;
     void *scratch = nullptr;

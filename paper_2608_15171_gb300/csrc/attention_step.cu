@@ -14,10 +14,6 @@ namespace ppas {
 
 namespace {
 
-// Decode rows are split so that one step launches about this many CTAs
-// (one per SM).
-constexpr int64_t kDecodeTargetCtas = kPlanSms;
-
 // Throughput model behind the SMs the prefill kernel leaves to the decode
 // launch (measured on GB300): one item's KV tile (two q-heads x 128 queries x
 // 128 keys) takes about 2.06 us of one SM; next to a running prefill kernel
@@ -80,19 +76,31 @@ size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 }  // namespace
 
+cudaError_t prepare_current_device() {
+    {
+        std::lock_guard<std::mutex> lock(g_side_mutex);
+        if (!side_stream()) return cudaErrorInitializationError;
+    }
+    cudaError_t e = prepare_prefill();
+    if (e == cudaSuccess) e = prepare_decode();
+    return e;
+}
+
 int32_t device_sm_count() {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+    if (cudaGetDevice(&dev) != cudaSuccess) return kDefaultPlanSms;
     static std::atomic<int> cached[64] = {};
     if (dev >= 0 && dev < 64) {
         const int c = cached[dev].load(std::memory_order_relaxed);
         if (c) return c;
     }
     int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = kDefaultPlanSms;
     if (dev >= 0 && dev < 64) cached[dev].store(n, std::memory_order_relaxed);
     return n;
 }
+
+int32_t plan_sms() { return std::max(1, std::min(device_sm_count(), kMaxPrefillCtas)); }
 
 // K or V cache [num_blocks, n_kv_heads, 16, 128] bf16 viewed as rows of 128
 // elements; one TMA box = 16 rows (one page) x 64 columns.
@@ -139,8 +147,10 @@ bool encode_q_map(CUtensorMap *map, const void *q, int32_t total_q, int32_t n_q_
 }
 
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                       int32_t n_kv_heads, int32_t /*num_sms*/) {
+                       int32_t n_kv_heads, int32_t num_sms) {
     DecodePlan d;
+    // decode rows are split so that one step launches about one CTA per SM
+    const int64_t target_ctas = std::max(1, num_sms);
     int64_t total_pages = 0;  // over (row, kv-head) pairs
     for (int32_t s = 0; s < n_seqs; ++s)
         if (q_lens[s] == 1) {
@@ -148,12 +158,12 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
             total_pages += static_cast<int64_t>((ctx_lens[s] + kPage - 1) / kPage) * n_kv_heads;
         }
     if (d.rows.empty()) return d;
-    // each (row, kv-head) gets a share of kDecodeTargetCtas CTAs in proportion
+    // each (row, kv-head) gets a share of target_ctas CTAs in proportion
     // to its pages (largest remainders first), so one step fills one wave
     const size_t nr = d.rows.size();
     std::vector<int64_t> shares(nr);
     {
-        const int64_t per_head = std::max<int64_t>(1, kDecodeTargetCtas / n_kv_heads);
+        const int64_t per_head = std::max<int64_t>(1, target_ctas / n_kv_heads);
         int64_t given = 0;
         std::vector<std::pair<int64_t, size_t>> rem(nr);  // (remainder, row)
         for (size_t k = 0; k < nr; ++k) {
@@ -384,7 +394,7 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
 }
 
 int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                           int32_t n_kv_heads) {
+                           int32_t n_kv_heads, int32_t num_sms) {
     const int32_t hpc = n_q_heads / n_kv_heads >= 2 ? 2 : 1;
     const int64_t slots = n_q_heads / hpc;
     double units = 0.0, bytes = 0.0;  // prefill KV tiles x head slots, decode K/V bytes
@@ -405,9 +415,9 @@ int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t 
     // the rest; the smallest k that finishes the decode rows by the time the
     // prefill items are done:  k r T(k) >= bytes,  T(k) = units tau / (S - k)
     const double sm_time = units * kPrefillTileUs;
-    int32_t k = static_cast<int32_t>(std::ceil(bytes * kPlanSms / (kDecodeBytesPerSmUs * sm_time + bytes)));
+    int32_t k = static_cast<int32_t>(std::ceil(bytes * num_sms / (kDecodeBytesPerSmUs * sm_time + bytes)));
     k = std::min(k, static_cast<int32_t>(kDecodeBytesPerUs / kDecodeBytesPerSmUs));
-    return std::max(0, std::min(k, kPlanSms / 2));
+    return std::max(0, std::min(k, num_sms / 2));
 }
 
 size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
@@ -415,7 +425,7 @@ size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *
     if (n_seqs <= 0 || !q_lens || !ctx_lens || n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads) return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (q_lens[s] < 1 || ctx_lens[s] < q_lens[s]) return 0;
-    return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes();
+    return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, plan_sms()).total_bytes();
 }
 
 }  // namespace ppas
@@ -503,8 +513,9 @@ extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h
         return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return 0;
-    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
-    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0).total_bytes() +
+    const int32_t sms = plan_sms();
+    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
+    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms).total_bytes() +
            plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas).total_bytes();
 }
 
@@ -521,8 +532,9 @@ extern "C" int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_
     }
     if (n_seqs == 0) return 0;
     // the same plans as ppas_attention_step
-    const DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
-    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
+    const int32_t sms = plan_sms();
+    const DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
+    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
     PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
     if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
         pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false, n_ctas);
@@ -558,8 +570,9 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         }
     }
 
-    DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, 0);
-    const int32_t n_ctas = kPlanSms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
+    const int32_t sms = plan_sms();
+    DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
+    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
     PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
     // a workspace too small for the prefill splits runs the prefill tiles unsplit
     if (workspace_bytes < dp.total_bytes() + pf.total_bytes())

@@ -341,10 +341,15 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     }
 }
 
+static std::atomic<uint64_t> g_decode_smem_set{0};
+
+cudaError_t prepare_decode() {
+    return ensure_smem_limit(decode_attn_kernel, static_cast<int>(kSmemBytes), g_decode_smem_set);
+}
+
 cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p,
                           cudaStream_t st) {
-    static std::atomic<uint64_t> smem_set{0};
-    const cudaError_t e = ensure_smem_limit(decode_attn_kernel, static_cast<int>(kSmemBytes), smem_set);
+    const cudaError_t e = prepare_decode();
     if (e != cudaSuccess) return e;
     if (p.n_ctas <= 0) return cudaSuccess;
     decode_attn_kernel<<<p.n_ctas, kDecodeWarps * 32, kSmemBytes, st>>>(tm_k, tm_v, p);

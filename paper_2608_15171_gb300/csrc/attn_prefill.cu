@@ -669,10 +669,15 @@ cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st) {
     return cudaLaunchKernelEx(&l.cfg, prefill_merge_kernel, p);
 }
 
+static std::atomic<uint64_t> g_prefill_smem_set{0};
+
+cudaError_t prepare_prefill() {
+    return ensure_smem_limit(prefill_attn_kernel, static_cast<int>(kSmemBytes), g_prefill_smem_set);
+}
+
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
                            const PrefillParams &p, cudaStream_t st) {
-    static std::atomic<uint64_t> smem_set{0};
-    const cudaError_t e = ensure_smem_limit(prefill_attn_kernel, static_cast<int>(kSmemBytes), smem_set);
+    const cudaError_t e = prepare_prefill();
     if (e != cudaSuccess) return e;
     if (p.n_ctas <= 0) return cudaSuccess;
     PdlLaunch l(dim3(p.n_ctas), dim3(kThreads), kSmemBytes, st);

@@ -18,9 +18,9 @@ constexpr int kPage = PPAS_PAGE_TOKENS;        // tokens per KV block
 constexpr int kHeadDim = 128;                  // the only head size with kernels
 constexpr int kRowBytes = kHeadDim * 2;        // one bf16 K or V row
 constexpr int kPageBytes = kPage * kRowBytes;  // one (block, kv-head) page: 4 KB
-// SMs the step plans are made for (GB300).  A fixed number keeps every plan,
-// and so the workspace size, a pure function of the step's lengths.
-constexpr int32_t kPlanSms = 152;
+// SMs the step plans assume when no device can be queried (GB300); with a
+// device the plans are made for its SM count (plan_sms()).
+constexpr int32_t kDefaultPlanSms = 152;
 
 // ------------------------------------------------------------------ prefill
 // Rows with q_len > 1.  The kernel is persistent: one CTA per SM works
@@ -130,9 +130,10 @@ struct PrefillPlan {
 };
 
 // SMs the persistent prefill kernel leaves to the decode launch of the same
-// step (0 without decode rows or without prefill chunks)
+// step on a device of num_sms SMs (0 without decode rows or without prefill
+// chunks)
 int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                           int32_t n_kv_heads);
+                           int32_t n_kv_heads, int32_t num_sms);
 
 // n_ctas: CTAs (SMs) the persistent kernel may occupy; allow_split == false
 // keeps every unit whole (no workspace)
@@ -196,10 +197,16 @@ struct DecodePlan {
 size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
                           int32_t n_kv_heads);
 
+// decode splits for a device of num_sms SMs: one wave of CTAs where the
+// split-size limits allow it
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
                        int32_t n_kv_heads, int32_t num_sms);
 
 int32_t device_sm_count();
+// SMs the current device's step plans are made for: its SM count, at most
+// kMaxPrefillCtas (one persistent prefill CTA per SM); kDefaultPlanSms
+// without a device
+int32_t plan_sms();
 
 // ------------------------------------------------------------------ gate-up projection
 struct GateUpParams {
@@ -265,6 +272,13 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
 
 cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p,
                           cudaStream_t st);
+
+// One-time per-device set-up the launchers otherwise do lazily on first use:
+// the kernels' shared-memory limits and the side stream and events of mixed
+// steps (for the current device).
+cudaError_t prepare_prefill();
+cudaError_t prepare_decode();
+cudaError_t prepare_current_device();
 
 // tensor maps (driver entry point fetched at run time)
 bool encode_kv_map(CUtensorMap *map, const void *cache, int32_t num_blocks, int32_t n_kv_heads);

@@ -38,7 +38,7 @@ EXPORTED = ("ppas_sched_create", "ppas_sched_destroy", "ppas_sched_free_blocks",
             "ppas_status_string", "ppas_abi_version", "ppas_attention_step_noalloc",
             "ppas_debug_wait_timeout", "ppas_attention_kernel_count", "ppas_gateup_pack",
             "ppas_gateup_swiglu")
-PPAS_NOALLOC_SCRATCH_BYTES = 4 * 1024 * 1024
+PPAS_NOALLOC_SCRATCH_BYTES = 64 * 1024 * 1024
 
 
 class ppas_request(ctypes.Structure):

@@ -1,8 +1,8 @@
 // Checks the host plan of the split-K decode kernel against what the kernel
 // indexes: for every case read from stdin
-//   <n_q_heads> <n_kv_heads> <n_seqs> <q_len>... <ctx_len>...
-// it plans the step's decode rows the way the attention call does and
-// verifies that
+//   <sms> <n_q_heads> <n_kv_heads> <n_seqs> <q_len>... <ctx_len>...
+// it plans the step's decode rows the way the attention call does on a
+// device of <sms> SMs and verifies that
 //  * the decode rows are exactly the rows with q_len == 1, in order;
 //  * split sp of a row covers pages [sp * pps, min((sp + 1) * pps, pages)),
 //    every split holds at least one page and the splits cover the row's
@@ -23,10 +23,10 @@
 
 using namespace ppas;
 
-static std::string check(int hq, int hk, const std::vector<int32_t> &q, const std::vector<int32_t> &c,
+static std::string check(int sms, int hq, int hk, const std::vector<int32_t> &q, const std::vector<int32_t> &c,
                          long long *ctas, long long *parts) {
     const int n = static_cast<int>(q.size());
-    DecodePlan d = plan_decode(n, q.data(), c.data(), hq, hk, 0);
+    DecodePlan d = plan_decode(n, q.data(), c.data(), hq, hk, sms);
     std::vector<int32_t> want;
     for (int s = 0; s < n; ++s)
         if (q[s] == 1) want.push_back(s);
@@ -55,13 +55,13 @@ static std::string check(int hq, int hk, const std::vector<int32_t> &q, const st
 }
 
 int main() {
-    int hq, hk, n;
-    while (std::cin >> hq >> hk >> n) {
+    int sms, hq, hk, n;
+    while (std::cin >> sms >> hq >> hk >> n) {
         std::vector<int32_t> q(n), c(n);
         for (auto &x : q) std::cin >> x;
         for (auto &x : c) std::cin >> x;
         long long ctas = 0, parts = 0;
-        const std::string err = check(hq, hk, q, c, &ctas, &parts);
+        const std::string err = check(sms, hq, hk, q, c, &ctas, &parts);
         if (!err.empty())
             std::printf("FAIL %s\n", err.c_str());
         else

@@ -1,7 +1,8 @@
 // Checks the host plan of the persistent prefill kernel against what the
 // kernel indexes: for every case read from stdin
-//   <n_q_heads> <n_kv_heads> <n_seqs> <q_len>... <ctx_len>...
-// it plans the step the way the attention call does and verifies that
+//   <sms> <n_q_heads> <n_kv_heads> <n_seqs> <q_len>... <ctx_len>...
+// it plans the step the way the attention call does on a device of <sms>
+// SMs and verifies that
 //  * each launch's tables (items, sequences, CTAs) fit their capacities and
 //    every CTA has at least one item;
 //  * every item's sequence, query tile, head slot and KV range are valid,
@@ -27,13 +28,13 @@
 
 using namespace ppas;
 
-static std::string check(int hq, int hk, const std::vector<int32_t> &q, const std::vector<int32_t> &c, bool split,
+static std::string check(int sms, int hq, int hk, const std::vector<int32_t> &q, const std::vector<int32_t> &c, bool split,
                          double *max_load, double *mean_load, size_t *n_launch, size_t *n_ctas, size_t *n_items,
                          long long *n_part) {
     const int n = static_cast<int>(q.size());
-    const int reserve = decode_reserve_sms(n, q.data(), c.data(), hq, hk);
-    if (reserve < 0 || reserve > kPlanSms / 2) return "reserve out of range";
-    const int avail = kPlanSms - reserve;
+    const int reserve = decode_reserve_sms(n, q.data(), c.data(), hq, hk, sms);
+    if (reserve < 0 || reserve > sms / 2) return "reserve out of range";
+    const int avail = sms - reserve;
     PrefillPlan pf = plan_prefill(n, q.data(), c.data(), hq, hk, split, avail);
     const int hpc = hq / hk >= 2 ? 2 : 1, slots = hq / hpc;
     if (pf.slots != slots || pf.heads_per_cta != hpc) return "head slots";
@@ -122,8 +123,8 @@ static std::string check(int hq, int hk, const std::vector<int32_t> &q, const st
 }
 
 int main() {
-    int hq, hk, n;
-    while (std::cin >> hq >> hk >> n) {
+    int sms, hq, hk, n;
+    while (std::cin >> sms >> hq >> hk >> n) {
         std::vector<int32_t> q(n), c(n);
         for (auto &x : q) std::cin >> x;
         for (auto &x : c) std::cin >> x;
@@ -131,7 +132,7 @@ int main() {
             double mx = 0, mean = 0;
             size_t nl = 0, nc = 0, ni = 0;
             long long np = 0;
-            const std::string err = check(hq, hk, q, c, split, &mx, &mean, &nl, &nc, &ni, &np);
+            const std::string err = check(sms, hq, hk, q, c, split, &mx, &mean, &nl, &nc, &ni, &np);
             if (!err.empty())
                 std::printf("FAIL %s%s\n", split ? "" : "(unsplit) ", err.c_str());
             else

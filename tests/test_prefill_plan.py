@@ -37,8 +37,8 @@ def checker(tmp_path_factory):
     return exe
 
 
-def _run(exe, cases):
-    text = "".join(f"{hq} {hk} {len(q)} " + " ".join(map(str, q)) + " " + " ".join(map(str, c)) + "\n"
+def _run(exe, cases, sms=152):
+    text = "".join(f"{sms} {hq} {hk} {len(q)} " + " ".join(map(str, q)) + " " + " ".join(map(str, c)) + "\n"
                    for hq, hk, q, c in cases)
     out = subprocess.run([exe], input=text, capture_output=True, text=True, check=True).stdout.split("\n")
     lines = [l for l in out if l]
@@ -59,9 +59,11 @@ def _paper_cases():
     return cases
 
 
-def test_paper_workloads_plan_valid_and_balanced(checker):
+@pytest.mark.parametrize("sms", [152, 148, 132])
+def test_paper_workloads_plan_valid_and_balanced(checker, sms):
+    """Plans for GB300's 152 SMs and for parts (or partitions) with fewer."""
     cases = _paper_cases()
-    res = _run(checker, [(g.n_q_heads, g.n_kv_heads, list(s.q_lens), list(s.ctx_lens)) for _, g, s in cases])
+    res = _run(checker, [(g.n_q_heads, g.n_kv_heads, list(s.q_lens), list(s.ctx_lens)) for _, g, s in cases], sms)
     for (name, _, _), (split, whole) in zip(cases, res):
         assert split.startswith("ok"), f"{name}: {split}"
         assert whole.startswith("ok"), f"{name}: {whole}"
@@ -71,7 +73,8 @@ def test_paper_workloads_plan_valid_and_balanced(checker):
             assert float(f[5]) <= 1.10 * float(f[6]), f"{name}: CTA loads {f[5]} vs mean {f[6]}"
 
 
-def test_random_steps_plan_valid(checker):
+@pytest.mark.parametrize("sms", [152, 132, 256])
+def test_random_steps_plan_valid(checker, sms):
     rng = np.random.default_rng(11)
     cases = []
     for _ in range(60):
@@ -92,6 +95,6 @@ def test_random_steps_plan_valid(checker):
     cases.append((32, 8, [128, 300], [65535 * 128 - 7, 4_000_000]))
     for kt in (511, 512, 513, 515, 516, 1024, 1025):
         cases.append((16, 2, [128], [kt * 128]))
-    for case, (split, whole) in zip(cases, _run(checker, cases)):
+    for case, (split, whole) in zip(cases, _run(checker, cases, sms)):
         assert split.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {split}"
         assert whole.startswith("ok"), f"{case[:2]} {len(case[2])} seqs: {whole}"
