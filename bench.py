@@ -819,7 +819,7 @@ def cpu_baseline(torch, args, device="cpu"):
             "kind": "oracle", "extrapolated": True,
             "sample": f"headline = config 2 ({head['kind']}, {head['seconds']} s) {head['extrapolated']}; "
                       f"oracle = float64 numpy, thread pool of {workers}, budget {budget:.0f} s",
-            "per_config": per}
+            "per_config": per, "planner": _planner_timing()}
 
 
 def _planner_timing():

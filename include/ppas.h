@@ -197,9 +197,12 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * Inside, when a step has both kinds of rows, the decode launch runs on a
  * library-owned side stream forked from `stream` (an event) and joined back
  * into it (a second event), so that it shares the GPU with the prefill
- * launch; the prefill and merge kernels are launched with programmatic
- * stream serialization (their set-up may overlap the kernel before them on
- * `stream`; every global-memory access waits for that kernel to complete).
+ * launch; the prefill, merge and decode kernels are launched with
+ * programmatic stream serialization (their set-up may overlap the kernel
+ * before them on their stream; every global-memory access waits for that
+ * kernel to complete).  The workspace needs no initialisation: the decode
+ * splits' arrival tickets in it carry a per-launch tag.  Plans, and so
+ * ppas_attention_workspace_size, follow the current device's SM count.
  * ------------------------------------------------------------------------- */
 size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
                                      const int32_t *h_ctx_lens, int32_t n_q_heads,
@@ -207,9 +210,10 @@ size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
 
 /* ---------------------------------------------------------------------------
  * Number of kernels ppas_attention_step launches for this step when given a
- * workspace of workspace_bytes (host only, no CUDA call): prefill launches,
- * the merge launch after each prefill launch whose plan cuts units, and
- * decode launches.  Memsets are not counted.  Returns -1 for arguments
+ * workspace of workspace_bytes (host only): prefill launches, the merge
+ * launch after each prefill launch whose plan cuts units, and decode
+ * launches, for the current device's plan (the call enqueues nothing else:
+ * no memset, no copy).  Returns -1 for arguments
  * ppas_attention_step would reject (see there); 0 for n_seqs == 0.
  * ------------------------------------------------------------------------- */
 int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
@@ -275,7 +279,8 @@ ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int
  *    call before any stream capture and before a phase in which nothing may
  *    be created.  PPAS_ERR_CUDA if the set-up fails.
  *  - All calls share one array, which keeps the last call's contents (the
- *    parts that must start at zero are cleared on the stream by every call).
+ *    decode split tickets in it carry a per-launch tag, so nothing in it has
+ *    to start at zero).
  *    Calls whose work overlaps on the GPU (other streams, other host threads)
  *    race on it: serialise them.
  * ------------------------------------------------------------------------- */

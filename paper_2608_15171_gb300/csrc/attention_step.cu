@@ -1,6 +1,7 @@
 // Host side of the C ABI: argument checks, TMA descriptors, the split of one
 // attention step into prefill tiles and decode splits, and the launches.
 #include <algorithm>
+#include <chrono>
 #include <cmath>
 #include <cstring>
 #include <mutex>
@@ -73,6 +74,18 @@ SideStream *side_stream() {
 }
 
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+// Tags of the decode launches' split tickets: never 0 and larger for every
+// launch of the process (the kernel relies on the order: a ticket word
+// holding a smaller tag is stale).  47 bits, so (tag << 16) | arrivals stays
+// below 2^63; the start is drawn from the clock so that tickets another
+// process left in recycled memory rarely match.
+unsigned long long next_launch_tag() {
+    static std::atomic<unsigned long long> next{
+        1 + ((static_cast<unsigned long long>(std::chrono::steady_clock::now().time_since_epoch().count()) *
+              0x9E3779B97F4A7C15ull) >> 24)};
+    return next.fetch_add(1, std::memory_order_relaxed) & ((1ull << 47) - 1);
+}
 
 }  // namespace
 
@@ -195,7 +208,7 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
     }
     d.ml_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * 2 * sizeof(float));
     d.o_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * kHeadDim * sizeof(float));
-    d.counter_bytes = align256(d.rows.size() * n_kv_heads * sizeof(int32_t));
+    d.counter_bytes = align256(d.rows.size() * n_kv_heads * sizeof(unsigned long long));
     return d;
 }
 
@@ -593,8 +606,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         uint8_t *ws = static_cast<uint8_t *>(workspace);
         float *part_ml = reinterpret_cast<float *>(ws);
         float *part_o = reinterpret_cast<float *>(ws + dp.ml_bytes);
-        int32_t *counters = reinterpret_cast<int32_t *>(ws + dp.ml_bytes + dp.o_bytes);
-        if (cudaMemsetAsync(counters, 0, dp.counter_bytes, ds) != cudaSuccess) return PPAS_ERR_CUDA;
+        auto *counters = reinterpret_cast<unsigned long long *>(ws + dp.ml_bytes + dp.o_bytes);
         DecodeParams dprm;
         std::memset(&dprm, 0, sizeof(dprm));
         dprm.q = static_cast<const __nv_bfloat16 *>(q);
@@ -630,6 +642,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
                 part_base += r.n_splits;
             }
             dprm.n_ctas = cta;
+            dprm.launch_tag = next_launch_tag();
             if (launch_decode(tm_k, tm_v, dprm, ds) != cudaSuccess) return PPAS_ERR_CUDA;
         }
         return PPAS_OK;

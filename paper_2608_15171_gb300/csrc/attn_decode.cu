@@ -14,6 +14,11 @@
 // partial goes to the workspace and the last CTA of the (row, kv-head) to
 // finish merges all splits:
 //   o = sum_i 2^(m_i - M) o_i / sum_i 2^(m_i - M) l_i,  M = max_i m_i.
+// The splits count their arrivals in a 64-bit ticket per (row, kv-head)
+// that carries the launch's tag (tags increase from launch to launch), so
+// tickets never need clearing before a launch; the kernel is launched with
+// programmatic stream serialization and touches global memory only after
+// grid_dep_wait().
 #include <math.h>
 
 #include "ppas_device.cuh"
@@ -97,6 +102,9 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
         fence_mbar_init();
     }
     if (tid == 0) *abort_flag = 0;
+    // the set-up above overlaps the kernel before this one on the stream;
+    // global memory (page ids, Q, pages, workspace, output) only after it
+    grid_dep_wait();
     // the split's page ids, loaded once by every thread in parallel
     for (int i = tid; i < pg1 - pg0; i += blockDim.x) ids[i] = __ldg(table + pg0 + i);
     __syncthreads();
@@ -270,10 +278,24 @@ __global__ void __launch_bounds__(kDecodeWarps * 32)
     __syncthreads();
     __shared__ int s_last;
     if (tid == 0) {
-        int *ctr = p.counters + lo * p.n_kv_heads + kvh;
-        const int prev = atomicAdd(ctr, 1);
+        // ticket = (tag << 16) | arrivals.  Tags grow from launch to launch, so
+        // atomicMax turns a word left by an earlier launch (or reset to 0)
+        // into this launch's tag with no arrivals, and leaves a word this
+        // launch already owns alone; only a word with a larger tag (memory
+        // nothing of this process wrote) is claimed by compare-and-swap.
+        // Then every split adds its arrival: two atomics, no retries.
+        unsigned long long *ctr = p.counters + lo * p.n_kv_heads + kvh;
+        const unsigned long long mine = p.launch_tag << 16;
+        unsigned long long cur = atomicMax(ctr, mine);
+        for (int it = 0; (cur >> 16) > p.launch_tag && it < (1 << 20); ++it) {
+            const unsigned long long got = atomicCAS(ctr, cur, mine);
+            cur = got == cur ? mine : got;
+        }
+        const unsigned long long old = atomicAdd(ctr, 1ull);
+        const int prev = (old >> 16) == p.launch_tag ? static_cast<int>(old & 0xFFFFull) : -1;
+        if (prev < 0) report_error(p.err, PPAS_DEVERR_TIMEOUT);  // the word was never claimed
         s_last = (prev == row.n_splits - 1);
-        if (s_last) *ctr = 0;  // ready for the next call
+        if (s_last) *ctr = 0;  // also ready for a replay with the same tag (a captured graph)
     }
     __syncthreads();
     if (!s_last) return;
@@ -352,8 +374,8 @@ cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, cons
     const cudaError_t e = prepare_decode();
     if (e != cudaSuccess) return e;
     if (p.n_ctas <= 0) return cudaSuccess;
-    decode_attn_kernel<<<p.n_ctas, kDecodeWarps * 32, kSmemBytes, st>>>(tm_k, tm_v, p);
-    return cudaGetLastError();
+    PdlLaunch l(dim3(p.n_ctas), dim3(kDecodeWarps * 32), kSmemBytes, st);
+    return cudaLaunchKernelEx(&l.cfg, decode_attn_kernel, tm_k, tm_v, p);
 }
 
 }  // namespace ppas

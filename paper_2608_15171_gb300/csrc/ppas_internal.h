@@ -176,7 +176,11 @@ struct DecodeParams {
     float scale_log2;
     float *part_ml;      // [n_part, n_q_heads, 2]   (m, l)
     float *part_o;       // [n_part, n_q_heads, 128] unnormalised
-    int32_t *counters;   // [n_rows, n_kv_heads]
+    // [n_rows, n_kv_heads] split tickets: (launch tag << 16) | arrivals; a
+    // word with an older tag counts as no arrival, and the last arriver
+    // resets its word to 0, so no call has to clear them
+    unsigned long long *counters;
+    unsigned long long launch_tag;  // 47 bits, never 0, larger for every launch
     int32_t *err;
     int32_t n_rows;
     int32_t n_ctas;

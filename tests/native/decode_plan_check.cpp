@@ -48,7 +48,7 @@ static std::string check(int sms, int hq, int hk, const std::vector<int32_t> &q,
     if (d.ml_bytes % 256 || d.o_bytes % 256 || d.counter_bytes % 256) return "alignment";
     if (d.ml_bytes < static_cast<size_t>(np) * hq * 2 * sizeof(float)) return "partial m/l bytes";
     if (d.o_bytes < static_cast<size_t>(np) * hq * kHeadDim * sizeof(float)) return "partial O bytes";
-    if (d.counter_bytes < d.rows.size() * hk * sizeof(int32_t)) return "ticket bytes";
+    if (d.counter_bytes < d.rows.size() * hk * sizeof(unsigned long long)) return "ticket bytes";
     *ctas = nc;
     *parts = np;
     return "";
