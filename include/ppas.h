@@ -6,7 +6,8 @@
  * plain host or device pointers and sizes; nothing here mentions a framework
  * type.  The library keeps no global state apart from per-device caches
  * (driver entry points, the SM count, the kernels' shared-memory limits, one
- * side stream with two events, all created on first use and thread-safe)
+ * side stream with two events for steps too large for one launch, all created
+ * on first use and thread-safe)
  * and the fixed scratch array of ppas_attention_step_noalloc; the only
  * stateful object is the opaque planner ppas_sched, which owns the free list
  * of KV blocks.
@@ -190,18 +191,26 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * (512 with group >= 2), ctx_len <= 65535*128 for rows with q_len > 1 and
  * ctx_len <= 2^25 for rows with q_len == 1; otherwise PPAS_ERR_UNSUPPORTED.  n_seqs == 0 is a no-op.  Block ids in the tables
  * must lie in [0, num_blocks) for every position below ctx_len.
- * Rows with q_len == 1 run on the split-K decode kernel; longer rows run on
- * the tcgen05 prefill kernel.
+ * Rows with q_len == 1 run as split-K decode work; longer rows run on the
+ * tcgen05 prefill path, whose long (query tile, head) units may be cut into
+ * pieces on several CTAs (when the workspace holds their partials) and
+ * merged by a short merge launch right after.
+ * Launches: a step with only decode rows is one decode launch; a step with
+ * prefill chunks is one launch of the prefill kernel, or, with decode rows
+ * as well, one mixed launch whose first CTAs run the prefill items and whose
+ * remaining CTAs run the decode splits; either is followed by the merge
+ * launch when its plan cuts units.  Only a step whose prefill items exceed
+ * one launch's tables (over 2200 items, 128 sequences, or with more than 112
+ * decode rows beside the chunks) takes several prefill launches; then the
+ * decode launch runs on a library-owned side stream forked from `stream`
+ * (an event) and joined back into it (a second event).
  * Stream semantics: all work is ordered after the work already on `stream`
  * and everything later on `stream` is ordered after it, as for one kernel.
- * Inside, when a step has both kinds of rows, the decode launch runs on a
- * library-owned side stream forked from `stream` (an event) and joined back
- * into it (a second event), so that it shares the GPU with the prefill
- * launch; the prefill, merge and decode kernels are launched with
- * programmatic stream serialization (their set-up may overlap the kernel
- * before them on their stream; every global-memory access waits for that
- * kernel to complete).  The workspace needs no initialisation: the decode
- * splits' arrival tickets in it carry a per-launch tag.  Plans, and so
+ * The kernels are launched with programmatic stream serialization (their
+ * set-up may overlap the kernel before them on their stream; every
+ * global-memory access waits for that kernel to complete).  The workspace
+ * needs no initialisation: the decode splits' arrival tickets in it carry a
+ * per-launch tag.  Plans, and so
  * ppas_attention_workspace_size, follow the current device's SM count.
  * ------------------------------------------------------------------------- */
 size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
@@ -210,10 +219,11 @@ size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
 
 /* ---------------------------------------------------------------------------
  * Number of kernels ppas_attention_step launches for this step when given a
- * workspace of workspace_bytes (host only): prefill launches, the merge
- * launch after each prefill launch whose plan cuts units, and decode
- * launches, for the current device's plan (the call enqueues nothing else:
- * no memset, no copy).  Returns -1 for arguments
+ * workspace of workspace_bytes (host only), for the current device's plan:
+ * its prefill (or mixed) launches, the merge launch after each one whose
+ * plan cuts units, and its decode launches unless they are part of a mixed
+ * launch (see ppas_attention_step; the call enqueues nothing else: no
+ * memset, no copy).  Returns -1 for arguments
  * ppas_attention_step would reject (see there); 0 for n_seqs == 0.
  * ------------------------------------------------------------------------- */
 int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
@@ -275,7 +285,8 @@ ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int
  *  - The first call on a device (with rows to run) does the library's
  *    one-time set-up for that device with it current: it looks up the
  *    array's device address, sets the kernels' shared-memory limits and
- *    creates the side stream and two events of mixed steps.  Make that first
+ *    creates the side stream and two events that steps too large for one
+ *    launch use.  Make that first
  *    call before any stream capture and before a phase in which nothing may
  *    be created.  PPAS_ERR_CUDA if the set-up fails.
  *  - All calls share one array, which keeps the last call's contents (the

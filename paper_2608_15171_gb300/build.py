@@ -63,7 +63,33 @@ def build(verbose: bool = False, extra=()) -> str:
     os.replace(tmp, LIB_PATH)
     if verbose:
         print(f"built {LIB_PATH}")
+    fast = _build_fast(verbose)
+    if verbose and fast is None:
+        print("note: _ppasfast not built (no Python headers); the binding uses ctypes for every call")
     return LIB_PATH
+
+
+def _build_fast(verbose: bool = False):
+    """The CPython module with the per-layer calls (csrc/pyfast.c), linked
+    against libppas.so; None when this Python has no headers to build it."""
+    import sysconfig
+    inc = sysconfig.get_paths().get("include")
+    if not inc or not os.path.exists(os.path.join(inc, "Python.h")):
+        return None
+    gcc = shutil.which("gcc") or shutil.which("cc")
+    if gcc is None:
+        return None
+    out = os.path.join(HERE, "_ppasfast" + (sysconfig.get_config_var("EXT_SUFFIX") or ".so"))
+    tmp = out + ".tmp"
+    cmd = [gcc, "-O2", "-shared", "-fPIC", f"-I{inc}", f"-I{INCLUDE}", os.path.join(CSRC, "pyfast.c"), "-o", tmp,
+           f"-L{HERE}", "-lppas", f"-Wl,-rpath,{HERE}"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"building _ppasfast failed:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, out)
+    if verbose:
+        print(f"built {out}")
+    return out
 
 
 if __name__ == "__main__":

@@ -4,6 +4,7 @@
 #include <chrono>
 #include <cmath>
 #include <cstring>
+#include <memory>
 #include <mutex>
 #include <vector>
 
@@ -96,6 +97,7 @@ cudaError_t prepare_current_device() {
     }
     cudaError_t e = prepare_prefill();
     if (e == cudaSuccess) e = prepare_decode();
+    if (e == cudaSuccess) e = prepare_mixed();
     return e;
 }
 
@@ -213,8 +215,9 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
 }
 
 PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas) {
+                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas, int32_t max_work) {
     PrefillPlan pf;
+    max_work = std::max(1, std::min(max_work, kMaxPrefillWork));
     const int32_t g = n_q_heads / n_kv_heads;
     pf.heads_per_cta = g >= 2 ? 2 : 1;
     pf.slots = n_q_heads / pf.heads_per_cta;
@@ -249,7 +252,7 @@ PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *c
         for (; u1 < units.size(); ++u1) {
             const bool new_seq = local[units[u1].seq] < 0;
             const int64_t pieces = (units[u1].n_kt + kPrefillMaxPiece - 1) / kPrefillMaxPiece;
-            if (min_items + pieces + n_ctas > kMaxPrefillWork) break;
+            if (min_items + pieces + n_ctas > max_work) break;
             if (new_seq && lp.seqs.size() == static_cast<size_t>(kMaxPrefillSeqs)) break;
             if (new_seq) {
                 local[units[u1].seq] = static_cast<int32_t>(lp.seqs.size());
@@ -441,6 +444,73 @@ size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *
     return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, plan_sms()).total_bytes();
 }
 
+
+// The plan of one step, shared by the workspace query, the launch count and
+// the step itself so that the three always agree: the decode splits, the
+// SMs left to the prefill kernel, and the prefill launches (with stream-K
+// cuts when the workspace holds their partials).  A step with both kinds of
+// rows whose prefill items fit one mixed launch runs as that single launch.
+StepPlan plan_step(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                   int32_t n_kv_heads, size_t workspace_bytes) {
+    StepPlan sp;
+    const int32_t sms = plan_sms();
+    sp.dp = plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, sms);
+    sp.n_ctas = sms - decode_reserve_sms(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, sms);
+    const bool may_mix = !sp.dp.rows.empty() && sp.dp.rows.size() <= static_cast<size_t>(kMaxMixedRows);
+    auto plan = [&](int32_t max_work) {
+        PrefillPlan pf = plan_prefill(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, true, sp.n_ctas, max_work);
+        // a workspace too small for the pieces' partials runs every unit whole
+        if (workspace_bytes < sp.dp.total_bytes() + pf.total_bytes())
+            pf = plan_prefill(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, false, sp.n_ctas, max_work);
+        return pf;
+    };
+    sp.pf = plan(may_mix ? kMaxMixedWork : kMaxPrefillWork);
+    sp.mixed = may_mix && sp.pf.launches.size() == 1;
+    if (may_mix && !sp.mixed) sp.pf = plan(kMaxPrefillWork);  // several prefill launches anyway
+    return sp;
+}
+
+namespace {
+
+// The last few plans made on this thread: every layer of a scheduler
+// iteration has the same step, so a serving loop plans it once per
+// iteration instead of once per layer (the stream-K search of a step like
+// MBT 2k takes ~70 us of host time).
+struct CachedPlan {
+    int32_t n = -1, hq = 0, hk = 0, sms = 0;
+    size_t ws = 0;
+    std::vector<int32_t> q, c;
+    std::shared_ptr<const StepPlan> plan;
+};
+constexpr int kPlanCache = 4;
+thread_local CachedPlan t_plans[kPlanCache];
+thread_local int t_plan_next = 0;
+
+}  // namespace
+
+std::shared_ptr<const StepPlan> plan_step_cached(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens,
+                                                 int32_t n_q_heads, int32_t n_kv_heads, size_t workspace_bytes) {
+    const int32_t sms = plan_sms();
+    for (const CachedPlan &e : t_plans)
+        if (e.plan && e.n == n_seqs && e.hq == n_q_heads && e.hk == n_kv_heads && e.sms == sms &&
+            e.ws == workspace_bytes && std::equal(q_lens, q_lens + n_seqs, e.q.begin()) &&
+            std::equal(ctx_lens, ctx_lens + n_seqs, e.c.begin()))
+            return e.plan;
+    auto sp = std::make_shared<const StepPlan>(
+        plan_step(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, workspace_bytes));
+    CachedPlan &e = t_plans[t_plan_next];
+    t_plan_next = (t_plan_next + 1) % kPlanCache;
+    e.n = n_seqs;
+    e.hq = n_q_heads;
+    e.hk = n_kv_heads;
+    e.sms = sms;
+    e.ws = workspace_bytes;
+    e.q.assign(q_lens, q_lens + n_seqs);
+    e.c.assign(ctx_lens, ctx_lens + n_seqs);
+    e.plan = sp;
+    return sp;
+}
+
 }  // namespace ppas
 
 using namespace ppas;
@@ -526,10 +596,7 @@ extern "C" size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h
         return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (h_q_lens[s] < 1 || h_ctx_lens[s] < h_q_lens[s]) return 0;
-    const int32_t sms = plan_sms();
-    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
-    return plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms).total_bytes() +
-           plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas).total_bytes();
+    return plan_step_cached(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, SIZE_MAX)->total_bytes();
 }
 
 extern "C" int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_q_lens, const int32_t *h_ctx_lens,
@@ -544,18 +611,66 @@ extern "C" int32_t ppas_attention_kernel_count(int32_t n_seqs, const int32_t *h_
         if (h_q_lens[s] == 1 && h_ctx_lens[s] > kMaxDecodeCtx) return -1;
     }
     if (n_seqs == 0) return 0;
-    // the same plans as ppas_attention_step
-    const int32_t sms = plan_sms();
-    const DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
-    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
-    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
-    if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
-        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false, n_ctas);
-    int32_t n = static_cast<int32_t>((dp.rows.size() + kMaxDecodeRows - 1) / kMaxDecodeRows);
-    for (const PrefillLaunchPlan &lp : pf.launches)
+    // the same plan as ppas_attention_step
+    const auto spp = plan_step_cached(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, workspace_bytes);
+    const StepPlan &sp = *spp;
+    // the prefill (or mixed) launches, each followed by its merge launches
+    // when its plan cuts units, and the decode launches unless mixed in
+    int32_t n = sp.mixed ? 0 : static_cast<int32_t>((sp.dp.rows.size() + kMaxDecodeRows - 1) / kMaxDecodeRows);
+    for (const PrefillLaunchPlan &lp : sp.pf.launches)
         n += 1 + static_cast<int32_t>((lp.split_units.size() + kMaxMergeUnits - 1) / kMaxMergeUnits);
     return n;
 }
+
+namespace {
+
+// The prefill launch parameters of one planned launch (prefill or mixed).
+template <class P>
+void fill_prefill_params(P &pp, const PrefillPlan &pf, const PrefillLaunchPlan &lp, const std::vector<int32_t> &q_start,
+                         const int32_t *h_q_lens, const int32_t *h_ctx_lens, uint8_t *pws) {
+    for (size_t i = 0; i < lp.seqs.size(); ++i) {
+        const int32_t sq = lp.seqs[i];
+        pp.seqs[i] = {q_start[sq], h_q_lens[sq], h_ctx_lens[sq], sq};
+    }
+    std::memcpy(pp.work, lp.work.data(), lp.work.size() * sizeof(PrefillWork));
+    std::memcpy(pp.cta_begin, lp.cta_begin.data(), lp.cta_begin.size() * sizeof(uint16_t));
+    pp.n_ctas = static_cast<int32_t>(lp.cta_begin.size()) - 1;
+    if (pf.n_part > 0) {
+        pp.part_o = reinterpret_cast<float *>(pws);
+        pp.part_ml = reinterpret_cast<float *>(pws + pf.o_bytes);
+    }
+}
+
+// The merge launches of one prefill launch's cut units (none when it cuts none).
+bool launch_merges(const PrefillPlan &pf, const PrefillLaunchPlan &lp, const std::vector<int32_t> &q_start,
+                   const int32_t *h_q_lens, const float *part_o, const float *part_ml, void *out, int32_t out_fp32,
+                   int32_t n_q_heads, cudaStream_t st) {
+    static thread_local MergeParams mp;
+    for (size_t i0 = 0; i0 < lp.split_units.size(); i0 += kMaxMergeUnits) {
+        const size_t i1 = std::min(lp.split_units.size(), i0 + kMaxMergeUnits);
+        mp.part_o = part_o;
+        mp.part_ml = part_ml;
+        mp.out = out;
+        mp.out_fp32 = out_fp32;
+        mp.n_q_heads = n_q_heads;
+        mp.heads_per_cta = pf.heads_per_cta;
+        mp.n_units = static_cast<int32_t>(i1 - i0);
+        for (size_t i = i0; i < i1; ++i) {
+            const PrefillSplitUnit &su = lp.split_units[i];
+            MergeUnit &mu = mp.units[i - i0];
+            mu.out_row0 = q_start[su.seq] + su.qt * kTileQ;
+            mu.part = su.part;
+            mu.rows_valid = static_cast<uint16_t>(std::min(kTileQ, h_q_lens[su.seq] - su.qt * kTileQ));
+            mu.n_splits = static_cast<uint16_t>(su.n_splits);
+            mu.head0 = static_cast<uint16_t>(su.slot * pf.heads_per_cta);
+            mu.pad = 0;
+        }
+        if (launch_prefill_merge(mp, st) != cudaSuccess) return false;
+    }
+    return true;
+}
+
+}  // namespace
 
 extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, const void *v_cache,
                                            int32_t num_blocks, const int32_t *d_block_tables,
@@ -583,14 +698,11 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         }
     }
 
-    const int32_t sms = plan_sms();
-    DecodePlan dp = plan_decode(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
-    const int32_t n_ctas = sms - decode_reserve_sms(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, sms);
-    PrefillPlan pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, true, n_ctas);
-    // a workspace too small for the prefill splits runs the prefill tiles unsplit
-    if (workspace_bytes < dp.total_bytes() + pf.total_bytes())
-        pf = plan_prefill(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, false, n_ctas);
-    const size_t need = dp.total_bytes() + pf.total_bytes();
+    const auto spp = plan_step_cached(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads, workspace_bytes);
+    const StepPlan &sp = *spp;
+    const DecodePlan &dp = sp.dp;
+    const PrefillPlan &pf = sp.pf;
+    const size_t need = sp.total_bytes();
     if (need > 0) {
         if (!workspace || workspace_bytes < need) return PPAS_ERR_CAPACITY;
         if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return PPAS_ERR_INVALID_ARG;
@@ -601,14 +713,9 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         !encode_kv_map(&tm_v, v_cache, num_blocks, n_kv_heads))
         return PPAS_ERR_CUDA;
 
-    auto run_decode = [&](cudaStream_t ds) -> ppas_status {
-        if (dp.rows.empty()) return PPAS_OK;
-        uint8_t *ws = static_cast<uint8_t *>(workspace);
-        float *part_ml = reinterpret_cast<float *>(ws);
-        float *part_o = reinterpret_cast<float *>(ws + dp.ml_bytes);
-        auto *counters = reinterpret_cast<unsigned long long *>(ws + dp.ml_bytes + dp.o_bytes);
-        DecodeParams dprm;
-        std::memset(&dprm, 0, sizeof(dprm));
+    uint8_t *const ws = static_cast<uint8_t *>(workspace);
+    // the decode rows [b0, b1) of the plan as launch parameters
+    auto fill_decode = [&](auto &dprm, size_t b0, size_t b1, int32_t part_base) {
         dprm.q = static_cast<const __nv_bfloat16 *>(q);
         dprm.block_tables = d_block_tables;
         dprm.table_stride = max_blocks_per_seq;
@@ -619,30 +726,68 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
         dprm.n_kv_heads = n_kv_heads;
         dprm.group = g;
         dprm.scale_log2 = scale_log2;
-        dprm.part_ml = part_ml;
-        dprm.part_o = part_o;
+        dprm.part_ml = reinterpret_cast<float *>(ws);
+        dprm.part_o = reinterpret_cast<float *>(ws + dp.ml_bytes);
         dprm.err = d_err_flag;
+        dprm.n_rows = static_cast<int32_t>(b1 - b0);
+        dprm.counters = reinterpret_cast<unsigned long long *>(ws + dp.ml_bytes + dp.o_bytes) + b0 * n_kv_heads;
+        int32_t cta = 0;
+        for (size_t i = b0; i < b1; ++i) {
+            const int32_t s = dp.rows[i];
+            DecodeRow &r = dprm.rows[i - b0];
+            r.q_row = q_start[s];
+            r.ctx_len = h_ctx_lens[s];
+            r.table_row = s;
+            r.n_splits = dp.n_splits[i];
+            r.pages_per_split = dp.pages_per_split[i];
+            r.cta_base = cta;
+            r.part_base = part_base;
+            cta += r.n_splits * n_kv_heads;
+            part_base += r.n_splits;
+        }
+        dprm.n_ctas = cta;
+        dprm.launch_tag = next_launch_tag();
+        return part_base;
+    };
+    auto fill_prefill_common = [&](auto &pp) {
+        pp.block_tables = d_block_tables;
+        pp.table_stride = max_blocks_per_seq;
+        pp.num_blocks = num_blocks;
+        pp.out = out;
+        pp.out_fp32 = out_is_fp32 ? 1 : 0;
+        pp.n_q_heads = n_q_heads;
+        pp.n_kv_heads = n_kv_heads;
+        pp.group = g;
+        pp.heads_per_cta = pf.heads_per_cta;
+        pp.scale_log2 = scale_log2;
+        pp.err = d_err_flag;
+    };
+    uint8_t *const pws = ws + dp.total_bytes();
+    auto q_map = [&](CUtensorMap *tm) { return encode_q_map(tm, q, static_cast<int32_t>(total_q), n_q_heads); };
+
+    // ---------------- both kinds of rows in one launch
+    if (sp.mixed) {
+        CUtensorMap tm_q;
+        if (!q_map(&tm_q)) return PPAS_ERR_CUDA;
+        static thread_local MixedParams mp;  // ~32 KB: kept off the stack
+        std::memset(&mp, 0, sizeof(mp));
+        fill_prefill_common(mp.pf);
+        fill_prefill_params(mp.pf, pf, pf.launches[0], q_start, h_q_lens, h_ctx_lens, pws);
+        fill_decode(mp.dc, 0, dp.rows.size(), 0);
+        if (launch_mixed(tm_q, tm_k, tm_v, mp, cs) != cudaSuccess) return PPAS_ERR_CUDA;
+        return launch_merges(pf, pf.launches[0], q_start, h_q_lens, mp.pf.part_o, mp.pf.part_ml, out, mp.pf.out_fp32,
+                             n_q_heads, cs)
+                   ? PPAS_OK
+                   : PPAS_ERR_CUDA;
+    }
+
+    auto run_decode = [&](cudaStream_t ds) -> ppas_status {
+        static thread_local DecodeParams dprm;
         int32_t part_base = 0;
         for (size_t b0 = 0; b0 < dp.rows.size(); b0 += kMaxDecodeRows) {
             const size_t b1 = std::min(dp.rows.size(), b0 + kMaxDecodeRows);
-            dprm.n_rows = static_cast<int32_t>(b1 - b0);
-            dprm.counters = counters + b0 * n_kv_heads;
-            int32_t cta = 0;
-            for (size_t i = b0; i < b1; ++i) {
-                const int32_t s = dp.rows[i];
-                DecodeRow &r = dprm.rows[i - b0];
-                r.q_row = q_start[s];
-                r.ctx_len = h_ctx_lens[s];
-                r.table_row = s;
-                r.n_splits = dp.n_splits[i];
-                r.pages_per_split = dp.pages_per_split[i];
-                r.cta_base = cta;
-                r.part_base = part_base;
-                cta += r.n_splits * n_kv_heads;
-                part_base += r.n_splits;
-            }
-            dprm.n_ctas = cta;
-            dprm.launch_tag = next_launch_tag();
+            std::memset(&dprm, 0, sizeof(dprm));
+            part_base = fill_decode(dprm, b0, b1, part_base);
             if (launch_decode(tm_k, tm_v, dprm, ds) != cudaSuccess) return PPAS_ERR_CUDA;
         }
         return PPAS_OK;
@@ -651,8 +796,9 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     // decode rows alone: launch on the caller's stream
     if (pf.empty()) return run_decode(cs);
 
-    // with prefill chunks in the same step the decode launch is forked onto
-    // a side stream after the prefill launch and joined back
+    // prefill chunks over several launches (more items than one launch
+    // holds) with decode rows: the decode launch is forked onto a side
+    // stream after the first prefill launch is queued and joined back
     // (the side stream and its events are created, and used, under the lock)
     std::unique_lock<std::mutex> side_lock(g_side_mutex, std::defer_lock);
     if (!dp.rows.empty()) side_lock.lock();
@@ -668,57 +814,16 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
     // ---------------- prefill chunks
     {
         CUtensorMap tm_q;
-        if (!encode_q_map(&tm_q, q, static_cast<int32_t>(total_q), n_q_heads)) return PPAS_ERR_CUDA;
-        uint8_t *pws = static_cast<uint8_t *>(workspace) + dp.total_bytes();
-        PrefillParams pp;
-        std::memset(&pp, 0, sizeof(pp));
-        pp.block_tables = d_block_tables;
-        pp.table_stride = max_blocks_per_seq;
-        pp.num_blocks = num_blocks;
-        pp.out = out;
-        pp.out_fp32 = out_is_fp32 ? 1 : 0;
-        pp.n_q_heads = n_q_heads;
-        pp.n_kv_heads = n_kv_heads;
-        pp.group = g;
-        pp.heads_per_cta = pf.heads_per_cta;
-        pp.scale_log2 = scale_log2;
-        pp.err = d_err_flag;
-        if (pf.n_part > 0) {
-            pp.part_o = reinterpret_cast<float *>(pws);
-            pp.part_ml = reinterpret_cast<float *>(pws + pf.o_bytes);
-        }
-        MergeParams mp;
-        std::memset(&mp, 0, sizeof(mp));
-        mp.part_o = pp.part_o;
-        mp.part_ml = pp.part_ml;
-        mp.out = out;
-        mp.out_fp32 = pp.out_fp32;
-        mp.n_q_heads = n_q_heads;
-        mp.heads_per_cta = pf.heads_per_cta;
+        if (!q_map(&tm_q)) return PPAS_ERR_CUDA;
+        static thread_local PrefillParams pp;  // ~31 KB: kept off the stack
         for (const PrefillLaunchPlan &lp : pf.launches) {
-            for (size_t i = 0; i < lp.seqs.size(); ++i) {
-                const int32_t sq = lp.seqs[i];
-                pp.seqs[i] = {q_start[sq], h_q_lens[sq], h_ctx_lens[sq], sq};
-            }
-            std::memcpy(pp.work, lp.work.data(), lp.work.size() * sizeof(PrefillWork));
-            std::memcpy(pp.cta_begin, lp.cta_begin.data(), lp.cta_begin.size() * sizeof(uint16_t));
-            pp.n_ctas = static_cast<int32_t>(lp.cta_begin.size()) - 1;
+            std::memset(&pp, 0, sizeof(pp));
+            fill_prefill_common(pp);
+            fill_prefill_params(pp, pf, lp, q_start, h_q_lens, h_ctx_lens, pws);
             if (launch_prefill(tm_q, tm_k, tm_v, pp, cs) != cudaSuccess) return PPAS_ERR_CUDA;
-            // the split units' partials are merged once the launch is done
-            for (size_t i0 = 0; i0 < lp.split_units.size(); i0 += kMaxMergeUnits) {
-                const size_t i1 = std::min(lp.split_units.size(), i0 + kMaxMergeUnits);
-                mp.n_units = static_cast<int32_t>(i1 - i0);
-                for (size_t i = i0; i < i1; ++i) {
-                    const PrefillSplitUnit &su = lp.split_units[i];
-                    MergeUnit &mu = mp.units[i - i0];
-                    mu.out_row0 = q_start[su.seq] + su.qt * kTileQ;
-                    mu.part = su.part;
-                    mu.rows_valid = static_cast<uint16_t>(std::min(kTileQ, h_q_lens[su.seq] - su.qt * kTileQ));
-                    mu.n_splits = static_cast<uint16_t>(su.n_splits);
-                    mu.head0 = static_cast<uint16_t>(su.slot * pf.heads_per_cta);
-                }
-                if (launch_prefill_merge(mp, cs) != cudaSuccess) return PPAS_ERR_CUDA;
-            }
+            // the launch's cut units are merged once it is done
+            if (!launch_merges(pf, lp, q_start, h_q_lens, pp.part_o, pp.part_ml, out, pp.out_fp32, n_q_heads, cs))
+                return PPAS_ERR_CUDA;
         }
     }
     if (side) {

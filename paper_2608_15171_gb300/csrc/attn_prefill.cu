@@ -35,11 +35,15 @@
 // consecutive CTAs (stream-K): each piece writes its partial (m, l, O) to the
 // workspace, and prefill_merge_kernel, launched after this kernel, combines
 // the pieces of every cut unit.
+// The same CTA body serves the mixed step's single launch (mixed_attn_kernel
+// below), whose CTAs past the prefill ones run decode splits
+// (attn_decode_body.cuh).
 // The kernel is launched with programmatic stream serialization: its set-up
 // (TMEM allocation, barriers, tensor-map prefetch) overlaps the kernel before
 // it on the stream, and global memory is touched only after grid_dep_wait().
 #include <math.h>
 
+#include "attn_decode_body.cuh"
 #include "ppas_device.cuh"
 #include "ppas_internal.h"
 
@@ -168,8 +172,8 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 }
 
 // 32 consecutive output columns of one row, scaled by inv_l
-__device__ __forceinline__ void store_row32(const PrefillParams &p, int64_t orow, int c4, const float (&v)[32],
-                                            float inv_l) {
+template <class P>
+__device__ __forceinline__ void store_row32(const P &p, int64_t orow, int c4, const float (&v)[32], float inv_l) {
     if (p.out_fp32) {
         float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.out) + orow * kHeadDim + c4 * 32);
 #pragma unroll
@@ -194,7 +198,8 @@ struct ItemView {
     int kt0, n_kt;         // KV tiles [kt0, kt0 + n_kt)
 };
 
-__device__ __forceinline__ ItemView item_view(const PrefillParams &p, int w) {
+template <class P>
+__device__ __forceinline__ ItemView item_view(const P &p, int w) {
     const PrefillWork wk = p.work[w];
     const PrefillSeq sq = p.seqs[wk.seq];
     ItemView v;
@@ -213,9 +218,10 @@ __device__ __forceinline__ int pages_in(int ctx_len, int j) {
 
 }  // namespace
 
-__global__ void __launch_bounds__(kThreads, 1)
-    prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                        const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ PrefillParams p) {
+// The work of prefill CTA `cta` of the plan in p (all 512 threads).
+template <class P>
+__device__ __forceinline__ void prefill_cta(const CUtensorMap &tm_q, const CUtensorMap &tm_k,
+                                            const CUtensorMap &tm_v, const P &p, int cta) {
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_s = smem_u32(smem_raw);
     const uint32_t sb = (raw_s + 1023u) & ~1023u;  // 1024-aligned for the 128-byte swizzle
@@ -224,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int hpc = p.heads_per_cta;
     // this CTA's items, in order
-    const int w_beg = p.cta_begin[blockIdx.x], w_end = p.cta_begin[blockIdx.x + 1];
+    const int w_beg = p.cta_begin[cta], w_end = p.cta_begin[cta + 1];
 
     auto bar = [&](int i) { return sb + kOffBar + 8u * static_cast<uint32_t>(i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sg + kOffAbort);
@@ -603,6 +609,34 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+__global__ void __launch_bounds__(kThreads, 1)
+    prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                        const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ PrefillParams p) {
+    prefill_cta(tm_q, tm_k, tm_v, p, blockIdx.x);
+}
+
+// A whole mixed step in one launch: CTAs [0, p.pf.n_ctas) run the prefill
+// items, the CTAs after them the decode splits (one (row, kv-head, split)
+// each, on warps 0-7; warps 8-15 hand their registers to them and leave).
+// The block scheduler starts CTAs in index order, so the first wave holds
+// every prefill CTA and fills the SMs left to the decode rows.
+__global__ void __launch_bounds__(kThreads, 1)
+    mixed_attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                      const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ MixedParams p) {
+    if (static_cast<int>(blockIdx.x) < p.pf.n_ctas) {
+        prefill_cta(tm_q, tm_k, tm_v, p.pf, blockIdx.x);
+        return;
+    }
+    if ((threadIdx.x >> 5) >= kDecodeWarps) {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsSmall));
+        return;
+    }
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsLarge));
+    decode_cta<true>(tm_k, tm_v, p.dc, static_cast<int>(blockIdx.x) - p.pf.n_ctas);
+}
+static_assert(kDecodeThreads == 8 * 32 && kDecodeSmemBytes <= kSmemBytes,
+              "decode CTAs of a mixed launch: warps 0-7 of the CTA, within its shared memory");
+
 // Combines the pieces of a split unit:
 //   o = sum_i 2^(m_i - M) o_i / sum_i 2^(m_i - M) l_i,  M = max_i m_i
 // (m in log2 units), taking the pieces four at a time with the running
@@ -670,9 +704,14 @@ cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st) {
 }
 
 static std::atomic<uint64_t> g_prefill_smem_set{0};
+static std::atomic<uint64_t> g_mixed_smem_set{0};
 
 cudaError_t prepare_prefill() {
     return ensure_smem_limit(prefill_attn_kernel, static_cast<int>(kSmemBytes), g_prefill_smem_set);
+}
+
+cudaError_t prepare_mixed() {
+    return ensure_smem_limit(mixed_attn_kernel, static_cast<int>(kSmemBytes), g_mixed_smem_set);
 }
 
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
@@ -682,6 +721,16 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
     if (p.n_ctas <= 0) return cudaSuccess;
     PdlLaunch l(dim3(p.n_ctas), dim3(kThreads), kSmemBytes, st);
     return cudaLaunchKernelEx(&l.cfg, prefill_attn_kernel, tm_q, tm_k, tm_v, p);
+}
+
+cudaError_t launch_mixed(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
+                         const MixedParams &p, cudaStream_t st) {
+    const cudaError_t e = prepare_mixed();
+    if (e != cudaSuccess) return e;
+    const int grid = p.pf.n_ctas + p.dc.n_ctas;
+    if (grid <= 0) return cudaSuccess;
+    PdlLaunch l(dim3(grid), dim3(kThreads), kSmemBytes, st);
+    return cudaLaunchKernelEx(&l.cfg, mixed_attn_kernel, tm_q, tm_k, tm_v, p);
 }
 
 }  // namespace ppas

@@ -77,6 +77,16 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t
     }
 }
 
+// ---------------------------------------------------------------- named barriers
+// bar.sync / bar.arrive on a named barrier (0 is __syncthreads); n counts
+// threads (a multiple of 32) and every warp taking part executes it as a
+// whole.  They have no time limit: callers keep every wait matched by
+// arrivals on all paths.
+__device__ __forceinline__ void nbar_sync(uint32_t id, uint32_t n) {
+    __syncwarp();
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int32_t x, int32_t y,
                                             uint32_t bar) {

@@ -8,6 +8,7 @@
 #include <stdint.h>
 
 #include <atomic>
+#include <memory>
 #include <vector>
 
 #include "ppas.h"
@@ -30,11 +31,11 @@ constexpr int32_t kDefaultPlanSms = 152;
 // first, and cuts the line into one equal segment per CTA (stream-K style),
 // so a unit is split only where a segment ends.  Each piece of a split unit
 // writes a partial (m, l, O) and a merge kernel launched after the prefill
-// kernel combines them.
+// (or mixed) launch combines them.
 constexpr int kTileQ = 128;             // query tokens per tile (tcgen05 M)
 constexpr int kPrefillKT = 128;         // keys per KV tile
 constexpr int kMaxPrefillSeqs = 128;    // per launch
-constexpr int kMaxPrefillWork = 2400;   // items per launch (bounded by the 32 KB parameter space)
+constexpr int kMaxPrefillWork = 2200;   // items per launch (bounded by the 32 KB parameter space)
 constexpr int kMaxPrefillCtas = 256;    // CTAs per launch (one per SM)
 constexpr int kPrefillItemCost = 3;     // per-item overhead (Q load, pipeline fill, epilogue), in KV tiles
 constexpr int kPrefillMinPiece = 4;     // shortest piece of a split unit, in KV tiles
@@ -62,7 +63,8 @@ struct PrefillWork {     // one item: (sequence, q tile, head slot, KV range)
 };
 static_assert(sizeof(PrefillWork) == 12, "compact work item");
 
-struct PrefillParams {
+template <int kWork>
+struct PrefillParamsT {
     const int32_t *block_tables;
     int32_t table_stride;
     int32_t num_blocks;
@@ -76,15 +78,16 @@ struct PrefillParams {
     int32_t *err;
     float *part_o;          // [n_part, heads_per_cta, 4 chunks, 128 rows, 32]
     float *part_ml;         // [n_part, heads_per_cta, 128 rows, 2]
-    int32_t n_ctas;         // grid size
+    int32_t n_ctas;         // CTAs running prefill items
     uint16_t cta_begin[kMaxPrefillCtas + 1];  // CTA c runs work[cta_begin[c] .. cta_begin[c + 1])
-    PrefillWork work[kMaxPrefillWork];
+    PrefillWork work[kWork];
     PrefillSeq seqs[kMaxPrefillSeqs];
 };
+using PrefillParams = PrefillParamsT<kMaxPrefillWork>;
 static_assert(sizeof(PrefillParams) + 3 * 128 <= 32764, "kernel parameter space");
 
-// Merge of the split units' partials, launched after the prefill kernel:
-// one thread per (split unit, head of the slot, query row, 4 columns).
+// Merge of the split units' partials, launched after the prefill (or mixed)
+// launch: one thread per (split unit, head of the slot, query row, 4 columns).
 constexpr int kMaxMergeUnits = 1024;  // split units per merge launch
 
 struct MergeUnit {
@@ -136,9 +139,10 @@ int32_t decode_reserve_sms(int32_t n_seqs, const int32_t *q_lens, const int32_t 
                            int32_t n_kv_heads, int32_t num_sms);
 
 // n_ctas: CTAs (SMs) the persistent kernel may occupy; allow_split == false
-// keeps every unit whole (no workspace)
+// keeps every unit whole (no workspace); max_work: items a launch may take
+// (kMaxMixedWork for a step that may run as one mixed launch)
 PrefillPlan plan_prefill(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas);
+                         int32_t n_kv_heads, bool allow_split, int32_t n_ctas, int32_t max_work = kMaxPrefillWork);
 
 // ------------------------------------------------------------------ decode
 // Rows with q_len == 1.  One CTA handles one (row, kv-head, split): the
@@ -163,7 +167,8 @@ struct DecodeRow {
     int32_t part_base;   // first partial slot (units of splits) of this row
 };
 
-struct DecodeParams {
+template <int kRows>
+struct DecodeParamsT {
     const __nv_bfloat16 *q;
     const int32_t *block_tables;
     int32_t table_stride;
@@ -184,8 +189,21 @@ struct DecodeParams {
     int32_t *err;
     int32_t n_rows;
     int32_t n_ctas;
-    DecodeRow rows[kMaxDecodeRows];
+    DecodeRow rows[kRows];
 };
+using DecodeParams = DecodeParamsT<kMaxDecodeRows>;
+
+// ------------------------------------------------------------------ mixed step
+// A step with both kinds of rows runs as one launch when its plan fits these
+// tables (the prefill items of one launch and up to kMaxMixedRows decode
+// rows): CTAs [0, pf.n_ctas) run prefill items, the rest decode splits.
+constexpr int kMaxMixedWork = kMaxPrefillWork;  // prefill items of a mixed launch
+constexpr int kMaxMixedRows = 112;              // decode rows of a mixed launch (the rest of the 32 KB)
+struct MixedParams {
+    PrefillParamsT<kMaxMixedWork> pf;
+    DecodeParamsT<kMaxMixedRows> dc;
+};
+static_assert(sizeof(MixedParams) + 3 * 128 <= 32764, "kernel parameter space");
 
 struct DecodePlan {
     std::vector<int32_t> rows;       // indices of q_len == 1 rows
@@ -196,6 +214,21 @@ struct DecodePlan {
     size_t ml_bytes = 0, o_bytes = 0, counter_bytes = 0;
     size_t total_bytes() const { return ml_bytes + o_bytes + counter_bytes; }
 };
+
+struct StepPlan {
+    DecodePlan dp;
+    PrefillPlan pf;
+    int32_t n_ctas = 0;   // SMs the prefill launches may occupy
+    bool mixed = false;   // prefill and decode rows in one launch
+    size_t total_bytes() const { return dp.total_bytes() + pf.total_bytes(); }
+};
+// the plan of a step given the caller's workspace (SIZE_MAX: as large as it needs)
+StepPlan plan_step(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
+                   int32_t n_kv_heads, size_t workspace_bytes);
+// the same, from a small per-thread cache of the last plans (a step is
+// planned once for all the layers that run it)
+std::shared_ptr<const StepPlan> plan_step_cached(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens,
+                                                 int32_t n_q_heads, int32_t n_kv_heads, size_t workspace_bytes);
 
 // workspace the step needs without prefill splits (decode partials only)
 size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
@@ -273,6 +306,9 @@ cudaError_t launch_kv_append(const void *k_new, const void *v_new, const int32_t
 cudaError_t launch_prefill_merge(const MergeParams &p, cudaStream_t st);
 cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
                            const PrefillParams &p, cudaStream_t st);
+// one launch of a mixed step: p.pf.n_ctas prefill CTAs, then p.dc.n_ctas decode CTAs
+cudaError_t launch_mixed(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
+                         const MixedParams &p, cudaStream_t st);
 
 cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p,
                           cudaStream_t st);
@@ -282,6 +318,7 @@ cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, cons
 // steps (for the current device).
 cudaError_t prepare_prefill();
 cudaError_t prepare_decode();
+cudaError_t prepare_mixed();
 cudaError_t prepare_current_device();
 
 // tensor maps (driver entry point fetched at run time)

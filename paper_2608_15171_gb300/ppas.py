@@ -21,6 +21,13 @@ LIB_PATH = os.path.join(_HERE, "libppas.so")
 if not os.path.exists(LIB_PATH):
     raise ImportError(f"{LIB_PATH} is missing: run paper_2608_15171_gb300.build.build() first")
 _lib = ctypes.CDLL(LIB_PATH)
+try:
+    # the per-layer calls through the CPython module (built beside the library
+    # when this Python has headers): same C entry points, ~1 us of argument
+    # parsing instead of ctypes' ~12 us
+    from . import _ppasfast as _fast
+except ImportError:
+    _fast = None
 
 PPAS_OK = 0
 PPAS_ERR_INVALID_ARG = -1
@@ -75,9 +82,10 @@ _lib.ppas_plan_step.restype = _c.c_int32
 _lib.ppas_kv_append.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_void_p,
                                 _c.c_int32, _c.c_int32, _c.c_int32, _c.c_void_p, _c.c_void_p]
 _lib.ppas_kv_append.restype = _c.c_int32
-_lib.ppas_attention_workspace_size.argtypes = [_c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32]
+_lib.ppas_attention_workspace_size.argtypes = [_c.c_int32, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32]
 _lib.ppas_attention_workspace_size.restype = _c.c_size_t
-_lib.ppas_attention_kernel_count.argtypes = [_c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_size_t]
+_lib.ppas_attention_kernel_count.argtypes = [_c.c_int32, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32,
+                                              _c.c_size_t]
 _lib.ppas_attention_kernel_count.restype = _c.c_int32
 _lib.ppas_gateup_pack.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32, _c.c_void_p]
 _lib.ppas_gateup_pack.restype = _c.c_int32
@@ -85,12 +93,12 @@ _lib.ppas_gateup_swiglu.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_
                                     _c.c_void_p, _c.c_void_p]
 _lib.ppas_gateup_swiglu.restype = _c.c_int32
 _lib.ppas_attention_step.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p,
-                                     _c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_int32, _c.c_int32,
+                                     _c.c_int32, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32, _c.c_int32, _c.c_int32,
                                      _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p, _c.c_size_t,
                                      _c.c_void_p, _c.c_void_p]
 _lib.ppas_attention_step.restype = _c.c_int32
 _lib.ppas_attention_step_noalloc.argtypes = [_c.c_void_p, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_void_p,
-                                             _c.c_int32, _P32, _P32, _c.c_int32, _c.c_int32, _c.c_int32,
+                                             _c.c_int32, _c.c_void_p, _c.c_void_p, _c.c_int32, _c.c_int32, _c.c_int32,
                                              _c.c_int32, _c.c_float, _c.c_void_p, _c.c_int32, _c.c_void_p,
                                              _c.c_void_p]
 _lib.ppas_attention_step_noalloc.restype = _c.c_int32
@@ -119,6 +127,15 @@ def _i32(a) -> np.ndarray:
 
 def _p32(a: np.ndarray):
     return a.ctypes.data_as(_P32)
+
+
+def _addr(a: np.ndarray) -> int:
+    """Address of an int32 array's data (the cheap route for a writable
+    array; per-step calls pass small length arrays on every layer)."""
+    try:
+        return ctypes.addressof(ctypes.c_int32.from_buffer(a))
+    except (TypeError, ValueError):  # read-only or empty
+        return a.ctypes.data
 
 
 def _ptr(t) -> int:
@@ -170,6 +187,11 @@ def ppas_plan_step(handle, reqs, n_reqs: int, now_us: int, threshold: int, mbt_h
 
 def ppas_kv_append(k_new, v_new, d_slot_mapping, n_tokens: int, k_cache, v_cache, num_blocks: int,
                    n_kv_heads: int, head_dim: int, d_err_flag=None, stream=None) -> None:
+    if _fast is not None:
+        _check(_fast.kv_append(_ptr(k_new), _ptr(v_new), _ptr(d_slot_mapping), int(n_tokens), _ptr(k_cache),
+                               _ptr(v_cache), int(num_blocks), int(n_kv_heads), int(head_dim), _ptr(d_err_flag),
+                               _stream(stream)), "ppas_kv_append")
+        return
     _check(_lib.ppas_kv_append(_ptr(k_new), _ptr(v_new), _ptr(d_slot_mapping), int(n_tokens), _ptr(k_cache),
                                _ptr(v_cache), int(num_blocks), int(n_kv_heads), int(head_dim), _ptr(d_err_flag),
                                _stream(stream)), "ppas_kv_append")
@@ -177,7 +199,7 @@ def ppas_kv_append(k_new, v_new, d_slot_mapping, n_tokens: int, k_cache, v_cache
 
 def ppas_attention_workspace_size(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: int) -> int:
     ql, cl = _i32(q_lens), _i32(ctx_lens)
-    return int(_lib.ppas_attention_workspace_size(int(ql.size), _p32(ql), _p32(cl), int(n_q_heads),
+    return int(_lib.ppas_attention_workspace_size(int(ql.size), _addr(ql), _addr(cl), int(n_q_heads),
                                                   int(n_kv_heads)))
 
 
@@ -194,7 +216,7 @@ def ppas_gateup_swiglu(x, w_packed, y, n_tokens: int, hidden: int, inter: int, d
 
 def ppas_attention_kernel_count(q_lens, ctx_lens, n_q_heads: int, n_kv_heads: int, workspace_bytes: int) -> int:
     ql, cl = _i32(q_lens), _i32(ctx_lens)
-    n = int(_lib.ppas_attention_kernel_count(int(ql.size), _p32(ql), _p32(cl), int(n_q_heads), int(n_kv_heads),
+    n = int(_lib.ppas_attention_kernel_count(int(ql.size), _addr(ql), _addr(cl), int(n_q_heads), int(n_kv_heads),
                                              int(workspace_bytes)))
     if n < 0:
         raise PpasError(PPAS_ERR_INVALID_ARG, "ppas_attention_kernel_count")
@@ -206,8 +228,15 @@ def ppas_attention_step(q, k_cache, v_cache, num_blocks: int, d_block_tables, ma
                         out_is_fp32: bool, workspace=None, workspace_bytes: int = 0, d_err_flag=None,
                         stream=None) -> None:
     ql, cl = _i32(q_lens), _i32(ctx_lens)
+    if _fast is not None:
+        _check(_fast.attention_step(_ptr(q), _ptr(k_cache), _ptr(v_cache), int(num_blocks), _ptr(d_block_tables),
+                                    int(max_blocks_per_seq), ql, cl, int(n_q_heads), int(n_kv_heads),
+                                    int(head_dim), float(scale), _ptr(out), 1 if out_is_fp32 else 0,
+                                    _ptr(workspace), int(workspace_bytes), _ptr(d_err_flag), _stream(stream)),
+               "ppas_attention_step")
+        return
     _check(_lib.ppas_attention_step(_ptr(q), _ptr(k_cache), _ptr(v_cache), int(num_blocks),
-                                    _ptr(d_block_tables), int(max_blocks_per_seq), _p32(ql), _p32(cl),
+                                    _ptr(d_block_tables), int(max_blocks_per_seq), _addr(ql), _addr(cl),
                                     int(ql.size), int(n_q_heads), int(n_kv_heads), int(head_dim),
                                     float(scale), _ptr(out), 1 if out_is_fp32 else 0, _ptr(workspace),
                                     int(workspace_bytes), _ptr(d_err_flag), _stream(stream)),
@@ -222,7 +251,7 @@ def ppas_attention_step_noalloc(q, k_cache, v_cache, num_blocks: int, d_block_ta
     ``PPAS_NOALLOC_SCRATCH_BYTES`` (shared by every call; serialise calls)."""
     ql, cl = _i32(q_lens), _i32(ctx_lens)
     _check(_lib.ppas_attention_step_noalloc(_ptr(q), _ptr(k_cache), _ptr(v_cache), int(num_blocks),
-                                            _ptr(d_block_tables), int(max_blocks_per_seq), _p32(ql), _p32(cl),
+                                            _ptr(d_block_tables), int(max_blocks_per_seq), _addr(ql), _addr(cl),
                                             int(ql.size), int(n_q_heads), int(n_kv_heads), int(head_dim),
                                             float(scale), _ptr(out), 1 if out_is_fp32 else 0, _ptr(d_err_flag),
                                             _stream(stream)),

@@ -117,12 +117,23 @@ def test_kernel_count_follows_the_plan(ppas):
     assert ws > 0
     assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, ws) == 2
     assert ppas.ppas_attention_kernel_count(it2.q_lens, it2.ctx_lens, 16, 2, 0) == 1
-    # decode rows alone: one decode launch; with a chunk whose units are cut:
-    # decode, prefill and merge launches
+    # decode rows alone: one decode launch; decode rows with a chunk: one
+    # mixed launch, and its merge launch when the plan cuts units
     assert ppas.ppas_attention_kernel_count([1, 1], [3000, 5000], 16, 2, 1 << 30) == 1
-    assert ppas.ppas_attention_kernel_count([1, 1, 512], [3000, 5000, 9000], 16, 2, 1 << 30) == 3
-    # more sequences than one launch holds (whole units): two prefill launches
+    assert ppas.ppas_attention_kernel_count([1, 1, 512], [3000, 5000, 9000], 16, 2, 1 << 30) == 2
+    assert ppas.ppas_attention_kernel_count([1, 1, 512], [3000, 5000, 9000], 16, 2, 0) == 1
+    # the paper's mixed workloads: the MBT 16k Llama step (whole units) is one
+    # launch; the MBT 2k steps cut units to balance the SMs (mixed + merge)
+    for shape, hq, hk, n in ((wl.high_pressure_step(0), 16, 2, 2), (wl.llama_hi_step(0), 32, 8, 1),
+                             (wl.llama_lo_step(0), 32, 8, 2)):
+        ws = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, hq, hk)
+        assert ppas.ppas_attention_kernel_count(shape.q_lens, shape.ctx_lens, hq, hk, ws) == n
+        assert ppas.ppas_attention_kernel_count(shape.q_lens, shape.ctx_lens, hq, hk, 0) == 1
+    # more sequences than one launch holds (whole units): two prefill launches,
+    # and with decode rows beside them a decode launch as well
     assert ppas.ppas_attention_kernel_count([200] * 150, [200 + 37 * i for i in range(150)], 16, 2, 1 << 30) == 2
+    assert ppas.ppas_attention_kernel_count([1] + [200] * 150, [900] + [200 + 37 * i for i in range(150)], 16, 2,
+                                            1 << 30) == 3
     assert ppas.ppas_attention_kernel_count([], [], 16, 2, 0) == 0
     with pytest.raises(ppas.PpasError):
         ppas.ppas_attention_kernel_count([0], [5], 16, 2, 0)

@@ -374,8 +374,8 @@ def test_full_size_sampled_rows(ppas, name, geo, mk):
 def test_full_layer_every_element(ppas, name, geo, mk):
     """One whole layer of every full-size workload, in the launch
     configuration the benchmark times (whole units or stream-K pieces with
-    their merge, decode rows on the side stream): every output element
-    against the float64 oracle."""
+    their merge; a mixed step's decode rows in the same launch as its
+    prefill tiles): every output element against the float64 oracle."""
     shape = mk()
     c = device_case(geo, shape, seed=2, extra_blocks=64)
     out = run_step(ppas, c, False)

@@ -1,6 +1,6 @@
 """Seeded random mixed steps against the float64 oracle: random group sizes,
 chunk lengths (ragged query tiles), prefixes (unaligned pages), decode rows,
-and both a full workspace (stream-K cuts, merge launches, split decode) and
+and both a full workspace (stream-K cuts and their merge, split decode) and
 none at all (whole-unit plans, no prefill splits).  All decode rows and
 sampled (token, head) rows of every chunk are compared."""
 import numpy as np

@@ -8,10 +8,11 @@ outputs and keeps its scratch in the library's fixed device array.
 These tests run it through the C ABI, two calls in a row each time, and check
 every output against the float64 oracle:
 
-* the MBT 2048 step (4 chunks + 8 multi-split decode rows), whose whole plan
-  (decode split partials and the prefill tiles' stream-K partials, merged by
-  the merge launch) fits the array: it must also equal the ordinary entry
-  point with a caller-owned workspace bit for bit (same plan);
+* the MBT 2048 step (4 chunks + 8 multi-split decode rows in one mixed
+  launch), whose whole plan (decode split partials and the prefill tiles'
+  stream-K partials, merged by the merge launch) fits the array: it must also
+  equal the ordinary entry point with a caller-owned workspace bit for bit
+  (same plan);
 * a 130-token chunk over a ~100k-token prefix plus a decode row, whose prefill
   units are longer than one piece may be and are always cut: the stream-K
   partials live in the fixed array beside the decode partials;
@@ -62,8 +63,8 @@ def test_noalloc_mbt2k_step_against_oracle_twice(ppas):
     shape = wl.high_pressure_step(0)          # 8 decode rows of ~25k context (several splits) + 4 chunks
     full = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads)
     assert 0 < full <= ppas.PPAS_NOALLOC_SCRATCH_BYTES
-    # prefill + merge of the cut units + decode, as with a full workspace
-    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == _kernels(ppas, shape, geo, full) == 3
+    # one mixed launch + the merge of the cut units, as with a full workspace
+    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == _kernels(ppas, shape, geo, full) == 2
     c = device_case(geo, shape, seed=5)
     want = oracle_full(c)
     ref = host64(run_step(ppas, c, out_fp32=True))
@@ -79,7 +80,7 @@ def test_noalloc_stream_k_pieces_in_the_fixed_array(ppas):
     full = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads)
     dec = ppas.ppas_attention_workspace_size([1], [25003], geo.n_q_heads, geo.n_kv_heads)
     assert dec < full <= ppas.PPAS_NOALLOC_SCRATCH_BYTES   # prefill partials beside the decode partials
-    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == 3   # prefill, merge, decode
+    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == 2   # mixed launch + merge
     c = device_case(geo, shape, seed=9)
     want = oracle_full(c)
     ref = host64(run_step(ppas, c, out_fp32=True))
@@ -94,8 +95,8 @@ def test_noalloc_prefill_unsplit_when_its_partials_do_not_fit(ppas):
     shape = wl.StepShape([1] + [1024] * 4, [25011] + [65536 + 1024] * 4)
     full = ppas.ppas_attention_workspace_size(shape.q_lens, shape.ctx_lens, geo.n_q_heads, geo.n_kv_heads)
     assert full > ppas.PPAS_NOALLOC_SCRATCH_BYTES
-    # without room for the pieces the plan keeps every unit whole: no merge
-    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == 2
+    # without room for the pieces the plan keeps every unit whole (one mixed launch)
+    assert _kernels(ppas, shape, geo, ppas.PPAS_NOALLOC_SCRATCH_BYTES) == 1
     c = device_case(geo, shape, seed=13)
     rows = sample_rows(shape, geo.n_q_heads, 48, seed=13)
     want = oracle_rows(c, rows)
