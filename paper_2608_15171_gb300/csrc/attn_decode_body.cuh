@@ -320,60 +320,57 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
     decode_cta_sync<kPartial>();
     if (!s_last) return;
     __threadfence();
-    // Every split's (m, l) in one round of loads, turned into weights
-    // w = 2^(m - M) / L per (split, head); then each thread sums one head's
-    // 4 columns over the splits, 16 independent float4 loads at a time.
-    // (The rings are free: the weights live where they were.)
+    // Warp hh merges head hh on its own (lane: 4 columns).  The first 16
+    // splits' O go out before the weights are known, so their latency hides
+    // that of the (m, l) round; the weights w = 2^(m - M) stay in a
+    // shared-memory row of the warp (the rings are free), 1 / L is applied
+    // at the end.
     const int ns = row.n_splits;
-    float *sw = reinterpret_cast<float *>(sg);            // [ns][kMaxGroup] m, then w
-    float *sl = sw + kMaxDecodeSplitsPerRow * kMaxGroup;  // [ns][kMaxGroup] l
-    for (int i = tid; i < ns * g; i += kDecodeThreads) {
-        const int s_ = i / g, hh = i - s_ * g;
-        const int64_t pi = static_cast<int64_t>(row.part_base + s_) * p.n_q_heads + kvh * g + hh;
-        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + pi * 2));
-        sw[s_ * kMaxGroup + hh] = ml.x;
-        sl[s_ * kMaxGroup + hh] = ml.y;
-    }
-    decode_cta_sync<kPartial>();
-    const int hh = tid >> 5, c4 = tid & 31;  // warp hh: head hh; lane: 4 columns
-    if (hh < g) {
-        float M = -INFINITY, L = 0.f;
-        for (int s_ = lane; s_ < ns; s_ += 32) M = fmaxf(M, sw[s_ * kMaxGroup + hh]);
-#pragma unroll
-        for (int o_ = 16; o_ >= 1; o_ >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o_));
-        for (int s_ = lane; s_ < ns; s_ += 32) {
-            const float m = sw[s_ * kMaxGroup + hh];
-            const float f = m == -INFINITY ? 0.f : ex2(m - M);
-            sw[s_ * kMaxGroup + hh] = f;
-            L += f * sl[s_ * kMaxGroup + hh];
-        }
-#pragma unroll
-        for (int o_ = 16; o_ >= 1; o_ >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o_);
-        const float inv_l = 1.f / L;
-        for (int s_ = lane; s_ < ns; s_ += 32) sw[s_ * kMaxGroup + hh] *= inv_l;
-    }
-    decode_cta_sync<kPartial>();
+    const int hh = warp, c4 = lane;
     if (hh >= g) return;
     const int head = kvh * g + hh;
     const float4 *po = reinterpret_cast<const float4 *>(p.part_o) + c4;
+    auto part_index = [&](int s_) { return static_cast<int64_t>(row.part_base + s_) * p.n_q_heads + head; };
+    float4 ov[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+        ov[k] = k < ns ? __ldcg(po + part_index(k) * (kHeadDim / 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
+    float *wm = reinterpret_cast<float *>(sg) + hh * 2 * kMaxDecodeSplitsPerRow;  // [ns] m, then w
+    float *wl = wm + kMaxDecodeSplitsPerRow;                                     // [ns] l
+    float M = -INFINITY;
+    for (int s_ = lane; s_ < ns; s_ += 32) {
+        const float2 ml = __ldcg(reinterpret_cast<const float2 *>(p.part_ml + part_index(s_) * 2));
+        wm[s_] = ml.x;
+        wl[s_] = ml.y;
+        M = fmaxf(M, ml.x);
+    }
+#pragma unroll
+    for (int o_ = 16; o_ >= 1; o_ >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o_));
+    float L = 0.f;
+    for (int s_ = lane; s_ < ns; s_ += 32) {
+        const float m = wm[s_];
+        const float f = m == -INFINITY ? 0.f : ex2(m - M);
+        wm[s_] = f;
+        L += f * wl[s_];
+    }
+#pragma unroll
+    for (int o_ = 16; o_ >= 1; o_ >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o_);
+    __syncwarp();
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int s0 = 0; s0 < ns; s0 += 16) {
-        float4 ov[16];
+        if (s0 > 0) {
 #pragma unroll
-        for (int k = 0; k < 16; ++k) {
-            if (s0 + k < ns) {
-                const int64_t pi = static_cast<int64_t>(row.part_base + s0 + k) * p.n_q_heads + head;
-                ov[k] = __ldcg(po + pi * (kHeadDim / 4));
-            } else {
-                ov[k] = make_float4(0.f, 0.f, 0.f, 0.f);
-            }
+            for (int k = 0; k < 16; ++k)
+                ov[k] = s0 + k < ns ? __ldcg(po + part_index(s0 + k) * (kHeadDim / 4)) : make_float4(0.f, 0.f, 0.f, 0.f);
         }
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-            const float f = s0 + k < ns ? sw[(s0 + k) * kMaxGroup + hh] : 0.f;
+            const float f = s0 + k < ns ? wm[s0 + k] : 0.f;
             acc = make_float4(acc.x + f * ov[k].x, acc.y + f * ov[k].y, acc.z + f * ov[k].z, acc.w + f * ov[k].w);
         }
     }
+    const float inv_l = 1.f / L;
+    acc = make_float4(acc.x * inv_l, acc.y * inv_l, acc.z * inv_l, acc.w * inv_l);
     const int64_t oi = (static_cast<int64_t>(row.q_row) * p.n_q_heads + head) * kHeadDim + 4 * c4;
     if (p.out_fp32) {
         *reinterpret_cast<float4 *>(static_cast<float *>(p.out) + oi) = acc;

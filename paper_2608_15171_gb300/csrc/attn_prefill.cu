@@ -479,9 +479,11 @@ __device__ __forceinline__ void prefill_cta(const CUtensorMap &tm_q, const CUten
                     for (int i = 0; i < kKT; ++i)
                         if (first_key + i > pos) s[i] = -INFINITY;
                 }
-                float mx0 = s[0], mx1 = s[1], mx2 = s[2], mx3 = s[3];
+                // four independent chains over the 128 scores, two new ones per max3
+                float mx0 = fmaxf(s[0], s[4]), mx1 = fmaxf(s[1], s[5]);
+                float mx2 = fmaxf(s[2], s[6]), mx3 = fmaxf(s[3], s[7]);
 #pragma unroll
-                for (int i = 4; i < kKT; i += 8) {
+                for (int i = 8; i < kKT; i += 8) {
                     mx0 = max3(mx0, s[i], s[i + 4]);
                     mx1 = max3(mx1, s[i + 1], s[i + 5]);
                     mx2 = max3(mx2, s[i + 2], s[i + 6]);
