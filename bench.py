@@ -201,6 +201,9 @@ def _low_step(torch, ppas, W, stream, timers=None, host=None):
                         ev = torch.cuda.Event()
                         ev.record(h2d)
                         landed.append(ev)
+            # every layer of the iteration launches the same kernels
+            launches += geo.n_layers * (1 + ppas.ppas_attention_kernel_count(st.q_len, st.ctx_len, hq, hk,
+                                                                              W.ws_bytes))
             for layer in range(geo.n_layers):
                 q, kn, vn, out = W.q[layer][it], W.kn[layer][it], W.vn[layer][it], W.out[layer][it]
                 if host is not None:
@@ -222,7 +225,6 @@ def _low_step(torch, ppas, W, stream, timers=None, host=None):
                     d2h.wait_stream(stream)
                     with torch.cuda.stream(d2h):
                         host["out"][it].copy_(out, non_blocking=True)
-                launches += 1 + ppas.ppas_attention_kernel_count(st.q_len, st.ctx_len, hq, hk, W.ws_bytes)
             if host is not None:
                 stream.wait_stream(h2d)
                 stream.wait_stream(d2h)
@@ -282,16 +284,16 @@ def _high_step(torch, ppas, W, stream, append=True):
     attention calls alone."""
     geo, sh = W.geo, W.shape
     hq, hk, D = geo.n_q_heads, geo.n_kv_heads, geo.head_dim
-    launches = 0
+    # the per-row lengths as the int32 arrays the calls take, once per step
+    ql, cl = np.asarray(sh.q_lens, dtype=np.int32), np.asarray(sh.ctx_lens, dtype=np.int32)
+    # every layer launches the same kernels
+    launches = geo.n_layers * ((1 if append else 0) + ppas.ppas_attention_kernel_count(ql, cl, hq, hk, W.ws_bytes))
     for layer in range(geo.n_layers):
         if append:
             ppas.ppas_kv_append(W.kn[layer], W.vn[layer], W.slots, sh.total_q, W.k_cache[layer],
                                 W.v_cache[layer], W.nb, hk, D, W.err, stream)
-            launches += 1
         ppas.ppas_attention_step(W.q[layer], W.k_cache[layer], W.v_cache[layer], W.nb, W.tables, W.width,
-                                 sh.q_lens, sh.ctx_lens, hq, hk, D, geo.scale, W.out[layer], False, W.ws, W.ws_bytes,
-                                 W.err, stream)
-        launches += ppas.ppas_attention_kernel_count(sh.q_lens, sh.ctx_lens, hq, hk, W.ws_bytes)
+                                 ql, cl, hq, hk, D, geo.scale, W.out[layer], False, W.ws, W.ws_bytes, W.err, stream)
     return launches
 
 
