@@ -5,7 +5,8 @@
  * The library is a plain shared object (libppas.so).  Every entry point takes
  * plain host or device pointers and sizes; nothing here mentions a framework
  * type.  The library keeps no global state apart from per-device caches
- * (driver entry points, the SM count, the kernels' shared-memory limits, one
+ * (driver entry points, the SM count, the kernels' shared-memory limits, how
+ * many decode thread-block clusters the device holds co-resident, one
  * side stream with two events for steps too large for one launch, all created
  * on first use and thread-safe)
  * and the fixed scratch array of ppas_attention_step_noalloc; the only
@@ -195,7 +196,10 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * tcgen05 prefill path, whose long (query tile, head) units may be cut into
  * pieces on several CTAs (when the workspace holds their partials) and
  * merged by a short merge launch right after.
- * Launches: a step with only decode rows is one decode launch; a step with
+ * Launches: a step with only decode rows is one decode launch (for a few
+ * rows on a device that holds enough of them co-resident, in thread-block
+ * clusters of 4 CTAs whose split partials merge through distributed shared
+ * memory before reaching the workspace); a step with
  * prefill chunks is one launch of the prefill kernel, or, with decode rows
  * as well, one mixed launch whose first CTAs run the prefill items and whose
  * remaining CTAs run the decode splits; either is followed by the merge
@@ -211,7 +215,8 @@ ppas_status ppas_kv_append(const void *k_new, const void *v_new, const int32_t *
  * global-memory access waits for that kernel to complete).  The workspace
  * needs no initialisation: the decode splits' arrival tickets in it carry a
  * per-launch tag.  Plans, and so
- * ppas_attention_workspace_size, follow the current device's SM count.
+ * ppas_attention_workspace_size, follow the current device's SM count (and,
+ * for steps of decode rows only, its cluster capacity).
  * ------------------------------------------------------------------------- */
 size_t ppas_attention_workspace_size(int32_t n_seqs, const int32_t *h_q_lens,
                                      const int32_t *h_ctx_lens, int32_t n_q_heads,

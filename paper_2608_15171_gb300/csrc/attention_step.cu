@@ -98,6 +98,7 @@ cudaError_t prepare_current_device() {
     cudaError_t e = prepare_prefill();
     if (e == cudaSuccess) e = prepare_decode();
     if (e == cudaSuccess) e = prepare_mixed();
+    if (e == cudaSuccess) decode_cluster_caps();  // the occupancy queries, once per device
     return e;
 }
 
@@ -162,10 +163,8 @@ bool encode_q_map(CUtensorMap *map, const void *q, int32_t total_q, int32_t n_q_
 }
 
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                       int32_t n_kv_heads, int32_t num_sms) {
+                       int32_t n_kv_heads, int32_t num_sms, const DecodeClusterCaps &caps) {
     DecodePlan d;
-    // decode rows are split so that one step launches about one CTA per SM
-    const int64_t target_ctas = std::max(1, num_sms);
     int64_t total_pages = 0;  // over (row, kv-head) pairs
     for (int32_t s = 0; s < n_seqs; ++s)
         if (q_lens[s] == 1) {
@@ -173,11 +172,13 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
             total_pages += static_cast<int64_t>((ctx_lens[s] + kPage - 1) / kPage) * n_kv_heads;
         }
     if (d.rows.empty()) return d;
-    // each (row, kv-head) gets a share of target_ctas CTAs in proportion
-    // to its pages (largest remainders first), so one step fills one wave
     const size_t nr = d.rows.size();
-    std::vector<int64_t> shares(nr);
-    {
+    // Splits of every row for target_ctas CTAs in clusters of c: each
+    // (row, kv-head) gets a share of them in proportion to its pages
+    // (largest remainders first), so one step fills one wave; with c > 1
+    // the shares are whole numbers of clusters.  False when c does not fit.
+    auto splits = [&](int64_t target_ctas, int32_t c, std::vector<int32_t> &ns_out, std::vector<int32_t> &pps_out) {
+        std::vector<int64_t> shares(nr);
         const int64_t per_head = std::max<int64_t>(1, target_ctas / n_kv_heads);
         int64_t given = 0;
         std::vector<std::pair<int64_t, size_t>> rem(nr);  // (remainder, row)
@@ -193,20 +194,62 @@ DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx
                              return a.first > b.first;
                          });
         for (size_t k = 0; k < nr && given < per_head; ++k, ++given) ++shares[rem[k].second];
+        ns_out.assign(nr, 0);
+        pps_out.assign(nr, 0);
+        for (size_t k = 0; k < nr; ++k) {
+            const int64_t pages = (ctx_lens[d.rows[k]] + kPage - 1) / kPage;
+            const int64_t share = c > 1 ? shares[k] / c * c : std::max<int64_t>(shares[k], 1);
+            if (share < 1) return false;
+            // even splits (the last one short by fewer than n_splits pages)
+            int64_t pps = (pages + share - 1) / share;
+            pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
+            pps = std::min<int64_t>(pps, kDecodeMaxPagesPerSplit);
+            int64_t ns = (pages + pps - 1) / pps;
+            if (c > 1) {
+                // a whole number of clusters; at most c - 1 of the splits are
+                // empty (past the row's pages), and the share is not exceeded
+                if (ns > share || ns <= share - c) return false;
+                ns = share;
+            }
+            ns_out[k] = static_cast<int32_t>(ns);
+            pps_out[k] = static_cast<int32_t>(pps);
+        }
+        return true;
+    };
+    std::vector<int32_t> ns1, pps1;
+    splits(std::max(1, num_sms), 1, ns1, pps1);
+    d.n_splits = ns1;
+    d.pages_per_split = pps1;
+    // Clusters of 4, for steps of decode rows only (a mixed launch keeps its
+    // grid free of them), when that plan still fills 15/16 of the SMs and
+    // streams at most 6 % more pages in its longest split than the plan
+    // without clusters.  The split merge's last CTA then reads a quarter of
+    // the partials, which is what bounds steps of a few rows.  (Clusters of
+    // 2, on a 4-row step, measured no faster and are not used.)
+    if (static_cast<int32_t>(nr) == n_seqs) {
+        int64_t max1 = 0;
+        for (size_t k = 0; k < nr; ++k) max1 = std::max<int64_t>(max1, pps1[k]);
+        const int32_t cs[1] = {4};
+        const int32_t cap[1] = {caps.ctas4};
+        for (int i = 0; i < 1; ++i) {
+            if (cap[i] < cs[i] || cap[i] > num_sms) continue;
+            std::vector<int32_t> ns, pps;
+            if (!splits(cap[i], cs[i], ns, pps)) continue;
+            int64_t ctas = 0, maxc = 0;
+            for (size_t k = 0; k < nr; ++k) {
+                ctas += static_cast<int64_t>(ns[k]) * n_kv_heads;
+                maxc = std::max<int64_t>(maxc, pps[k]);
+            }
+            if (ctas > cap[i] || ctas * 16 < static_cast<int64_t>(num_sms) * 15 || maxc * 100 > max1 * 106) continue;
+            d.n_splits = ns;
+            d.pages_per_split = pps;
+            d.cluster = cs[i];
+            break;
+        }
     }
     for (size_t k = 0; k < nr; ++k) {
-        const int32_t s = d.rows[k];
-        const int64_t pages = (ctx_lens[s] + kPage - 1) / kPage;
-        const int64_t share = std::max<int64_t>(shares[k], 1);
-        // even splits (the last one short by fewer than n_splits pages)
-        int64_t pps = (pages + share - 1) / share;
-        pps = std::max<int64_t>(pps, kDecodeMinPagesPerSplit);
-        pps = std::min<int64_t>(pps, kDecodeMaxPagesPerSplit);
-        const int32_t ns = static_cast<int32_t>((pages + pps - 1) / pps);
-        d.n_splits.push_back(ns);
-        d.pages_per_split.push_back(static_cast<int32_t>(pps));
-        d.n_part += ns;
-        d.n_ctas += static_cast<int64_t>(ns) * n_kv_heads;
+        d.n_part += d.n_splits[k] / d.cluster;
+        d.n_ctas += static_cast<int64_t>(d.n_splits[k]) * n_kv_heads;
     }
     d.ml_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * 2 * sizeof(float));
     d.o_bytes = align256(static_cast<size_t>(d.n_part) * n_q_heads * kHeadDim * sizeof(float));
@@ -441,7 +484,8 @@ size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *
     if (n_seqs <= 0 || !q_lens || !ctx_lens || n_q_heads < 1 || n_kv_heads < 1 || n_q_heads % n_kv_heads) return 0;
     for (int32_t s = 0; s < n_seqs; ++s)
         if (q_lens[s] < 1 || ctx_lens[s] < q_lens[s]) return 0;
-    return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, plan_sms()).total_bytes();
+    return plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, plan_sms(), decode_cluster_caps())
+        .total_bytes();
 }
 
 
@@ -454,7 +498,7 @@ StepPlan plan_step(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_len
                    int32_t n_kv_heads, size_t workspace_bytes) {
     StepPlan sp;
     const int32_t sms = plan_sms();
-    sp.dp = plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, sms);
+    sp.dp = plan_decode(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, sms, decode_cluster_caps());
     sp.n_ctas = sms - decode_reserve_sms(n_seqs, q_lens, ctx_lens, n_q_heads, n_kv_heads, sms);
     const bool may_mix = !sp.dp.rows.empty() && sp.dp.rows.size() <= static_cast<size_t>(kMaxMixedRows);
     auto plan = [&](int32_t max_work) {
@@ -743,7 +787,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
             r.cta_base = cta;
             r.part_base = part_base;
             cta += r.n_splits * n_kv_heads;
-            part_base += r.n_splits;
+            part_base += r.n_splits / dp.cluster;
         }
         dprm.n_ctas = cta;
         dprm.launch_tag = next_launch_tag();
@@ -788,7 +832,7 @@ extern "C" ppas_status ppas_attention_step(const void *q, const void *k_cache, c
             const size_t b1 = std::min(dp.rows.size(), b0 + kMaxDecodeRows);
             std::memset(&dprm, 0, sizeof(dprm));
             part_base = fill_decode(dprm, b0, b1, part_base);
-            if (launch_decode(tm_k, tm_v, dprm, ds) != cudaSuccess) return PPAS_ERR_CUDA;
+            if (launch_decode(tm_k, tm_v, dprm, dp.cluster, ds) != cudaSuccess) return PPAS_ERR_CUDA;
         }
         return PPAS_OK;
     };

@@ -37,13 +37,21 @@ constexpr uint32_t kRingBytes = kDecodeStages * kStageBytes;
 constexpr uint32_t kOffBar = kDecodeWarps * kRingBytes;
 constexpr uint32_t kOffFlag = kOffBar + kDecodeWarps * kDecodeStages * 8;
 constexpr uint32_t kOffIds = kOffFlag + 16;   // page ids of this split
-constexpr uint32_t kSmemBytes = kOffIds + kDecodeMaxPagesPerSplit * 4 + 1024;
+// a cluster's merge: rank 0's slots for the cluster's CTA partials
+// ([rank][group][128] O, then [rank][group][2] (m, l)), outside the rings,
+// which a slower CTA of the cluster may still be streaming through when a
+// faster one writes its partial
+constexpr int kMaxCluster = 4;
+constexpr uint32_t kOffClusterRecv = kOffIds + kDecodeMaxPagesPerSplit * 4;
+constexpr uint32_t kClusterRecvBytes = kMaxCluster * 8 * (kHeadDim + 2) * 4;
+constexpr uint32_t kSmemBytes = kOffClusterRecv + kClusterRecvBytes + 1024;
 static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 // merge scratch (aliases the rings once every warp is done)
 constexpr int kMaxGroup = 8;
 static_assert(kDecodeWarps * kMaxGroup * (2 + kHeadDim) * 4 <= static_cast<int>(kOffBar), "merge scratch");
 static_assert(2 * kMaxDecodeSplitsPerRow * kMaxGroup * 4 <= static_cast<int>(kOffBar), "split weights");
 static_assert(kDecodeWarps >= kMaxGroup, "the split merge gives each head of a group one warp");
+static_assert(kClusterRecvBytes == kMaxCluster * kMaxGroup * (kHeadDim + 2) * 4, "cluster slots");
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3) {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
@@ -90,6 +98,12 @@ __device__ __forceinline__ void decode_cta_sync() {
 // the CTA has more threads, which do not take part).
 template <bool kPartial, class P>
 __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const P &p, int bid) {
+    // in a cluster launch every CTA announces that it has started; the
+    // matching wait comes before the first store into another CTA's shared
+    // memory (the barrier phases of every CTA: this one, then one after
+    // the stores, on every path)
+    if constexpr (!kPartial)
+        if (cluster_nctarank() > 1) cluster_arrive_relaxed();
     using namespace decode_detail;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw_s = smem_u32(smem_raw);
@@ -260,7 +274,18 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
         for (int n = 0; n < 16; ++n) *reinterpret_cast<float2 *>(dst + n * 8 + 2 * c) = make_float2(o[n][0], o[n][1]);
     }
     decode_cta_sync<kPartial>();
-    if (*abort_flag) return;
+    // CTAs per thread-block cluster: 1 unless the launch groups the splits of
+    // a (row, kv-head) into clusters (steps of decode rows only)
+    const uint32_t nct = kPartial ? 1u : cluster_nctarank();
+    // (in a cluster an aborted CTA carries on to the cluster barrier below)
+    if (nct == 1 && *abort_flag) return;
+    // rank 0's slot for this CTA's partial (cluster launches only)
+    const uint32_t crank = nct > 1 ? cluster_ctarank() : 0u;
+    const uint32_t recv = sb + kOffClusterRecv;
+    const uint32_t slot_o = nct > 1 ? dsmem_addr(recv + crank * (kMaxGroup * kHeadDim * 4), 0) : 0u;
+    const uint32_t slot_ml =
+        nct > 1 ? dsmem_addr(recv + kMaxCluster * kMaxGroup * kHeadDim * 4 + crank * (kMaxGroup * 2 * 4), 0) : 0u;
+    if (nct > 1) cluster_wait();  // every CTA of the cluster has started (its arrive at entry)
 
     // thread -> (head-dim column, first head); the CTA's threads cover
     // kDecodeThreads / 128 heads at a time
@@ -273,7 +298,10 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
         float L = 0.f, O = 0.f;
 #pragma unroll
         for (int w = 0; w < kDecodeWarps; ++w) {
-            const float f = ex2(cm[w * kMaxGroup + hh] - M);
+            // a warp without keys (or a split past its row's pages, which a
+            // cluster plan may hold) has m = -inf and weight 0
+            const float m = cm[w * kMaxGroup + hh];
+            const float f = m == -INFINITY ? 0.f : ex2(m - M);
             L += f * cl[w * kMaxGroup + hh];
             O += f * co[(w * kMaxGroup + hh) * kHeadDim + t];
         }
@@ -282,6 +310,12 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
             const int64_t oi = (static_cast<int64_t>(row.q_row) * p.n_q_heads + head) * kHeadDim + t;
             if (p.out_fp32) static_cast<float *>(p.out)[oi] = O / L;
             else static_cast<__nv_bfloat16 *>(p.out)[oi] = __float2bfloat16_rn(O / L);
+        } else if (nct > 1) {
+            dsmem_st_f32(slot_o + static_cast<uint32_t>(hh * kHeadDim + t) * 4u, O);
+            if (t == 0) {
+                dsmem_st_f32(slot_ml + static_cast<uint32_t>(hh * 2) * 4u, M);
+                dsmem_st_f32(slot_ml + static_cast<uint32_t>(hh * 2 + 1) * 4u, L);
+            }
         } else {
             const int64_t pi = static_cast<int64_t>(row.part_base + sp) * p.n_q_heads + head;
             p.part_o[pi * kHeadDim + t] = O;
@@ -292,6 +326,40 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
         }
     }
     if (row.n_splits == 1) return;
+    int n_parts = row.n_splits;  // partial slots of this (row, kv-head)
+    if constexpr (!kPartial) {
+        if (nct > 1) {
+            // The cluster's CTAs are consecutive splits sp0 .. sp0 + nct - 1
+            // of this (row, kv-head) (sp0 a multiple of nct, rank = sp -
+            // sp0).  Each has stored its partial into rank 0's slots above;
+            // after the barrier (every CTA reaches it, an aborted one too)
+            // rank 0 merges them from its own shared memory into partial
+            // slot sp0 / nct, and the others are done.
+            cluster_sync_all();
+            if (crank != 0) return;
+            const float *ro = reinterpret_cast<const float *>(sg + kOffClusterRecv);
+            const float *rml = ro + kMaxCluster * kMaxGroup * kHeadDim;
+            for (int hh = tid / kHeadDim; hh < g; hh += hstep) {
+                float M = -INFINITY;
+                for (uint32_t r = 0; r < nct; ++r) M = fmaxf(M, rml[(r * kMaxGroup + hh) * 2]);
+                float L = 0.f, O = 0.f;
+                for (uint32_t r = 0; r < nct; ++r) {
+                    const float m = rml[(r * kMaxGroup + hh) * 2];
+                    const float f = m == -INFINITY ? 0.f : ex2(m - M);
+                    L += f * rml[(r * kMaxGroup + hh) * 2 + 1];
+                    O += f * ro[(r * kMaxGroup + hh) * kHeadDim + t];
+                }
+                const int64_t pi =
+                    static_cast<int64_t>(row.part_base + sp / static_cast<int>(nct)) * p.n_q_heads + kvh * g + hh;
+                p.part_o[pi * kHeadDim + t] = O;
+                if (t == 0) {
+                    p.part_ml[pi * 2] = M;
+                    p.part_ml[pi * 2 + 1] = L;
+                }
+            }
+            n_parts = row.n_splits / static_cast<int>(nct);
+        }
+    }
 
     // ---- the last CTA of this (row, kv-head) merges every split
     __threadfence();
@@ -314,7 +382,7 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
         const unsigned long long old = atomicAdd(ctr, 1ull);
         const int prev = (old >> 16) == p.launch_tag ? static_cast<int>(old & 0xFFFFull) : -1;
         if (prev < 0) report_error(p.err, PPAS_DEVERR_TIMEOUT);  // the word was never claimed
-        s_last = (prev == row.n_splits - 1);
+        s_last = (prev == n_parts - 1);
         if (s_last) *ctr = 0;  // also ready for a replay with the same tag (a captured graph)
     }
     decode_cta_sync<kPartial>();
@@ -325,7 +393,7 @@ __device__ __forceinline__ void decode_cta(const CUtensorMap &tm_k, const CUtens
     // that of the (m, l) round; the weights w = 2^(m - M) stay in a
     // shared-memory row of the warp (the rings are free), 1 / L is applied
     // at the end.
-    const int ns = row.n_splits;
+    const int ns = n_parts;
     const int hh = warp, c4 = lane;
     if (hh >= g) return;
     const int head = kvh * g + hh;

@@ -207,9 +207,14 @@ static_assert(sizeof(MixedParams) + 3 * 128 <= 32764, "kernel parameter space");
 
 struct DecodePlan {
     std::vector<int32_t> rows;       // indices of q_len == 1 rows
-    std::vector<int32_t> n_splits;   // per decode row
+    std::vector<int32_t> n_splits;   // per decode row (a multiple of cluster)
     std::vector<int32_t> pages_per_split;  // per decode row
-    int64_t n_part = 0;              // sum of splits
+    // CTAs per thread-block cluster of the decode launch: the splits of a
+    // (row, kv-head) come in groups of `cluster` consecutive CTAs that merge
+    // their partials through distributed shared memory, so one partial slot
+    // per group reaches the workspace (1: no clusters)
+    int32_t cluster = 1;
+    int64_t n_part = 0;              // partial slots: sum of splits / cluster
     int64_t n_ctas = 0;
     size_t ml_bytes = 0, o_bytes = 0, counter_bytes = 0;
     size_t total_bytes() const { return ml_bytes + o_bytes + counter_bytes; }
@@ -234,10 +239,18 @@ std::shared_ptr<const StepPlan> plan_step_cached(int32_t n_seqs, const int32_t *
 size_t workspace_min_size(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
                           int32_t n_kv_heads);
 
+// How many decode CTAs can be co-resident in clusters of 2 and of 4 (0: no
+// clusters, e.g. without a device).
+struct DecodeClusterCaps {
+    int32_t ctas2 = 0, ctas4 = 0;
+};
+DecodeClusterCaps decode_cluster_caps();  // the current device's, cached
+
 // decode splits for a device of num_sms SMs: one wave of CTAs where the
-// split-size limits allow it
+// split-size limits allow it.  A step of decode rows only may run its
+// splits in clusters (caps: what the device holds co-resident).
 DecodePlan plan_decode(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens, int32_t n_q_heads,
-                       int32_t n_kv_heads, int32_t num_sms);
+                       int32_t n_kv_heads, int32_t num_sms, const DecodeClusterCaps &caps = {});
 
 int32_t device_sm_count();
 // SMs the current device's step plans are made for: its SM count, at most
@@ -310,8 +323,9 @@ cudaError_t launch_prefill(const CUtensorMap &tm_q, const CUtensorMap &tm_k, con
 cudaError_t launch_mixed(const CUtensorMap &tm_q, const CUtensorMap &tm_k, const CUtensorMap &tm_v,
                          const MixedParams &p, cudaStream_t st);
 
+// cluster: CTAs per thread-block cluster (the plan's DecodePlan::cluster)
 cudaError_t launch_decode(const CUtensorMap &tm_k, const CUtensorMap &tm_v, const DecodeParams &p,
-                          cudaStream_t st);
+                          int32_t cluster, cudaStream_t st);
 
 // One-time per-device set-up the launchers otherwise do lazily on first use:
 // the kernels' shared-memory limits and the side stream and events of mixed

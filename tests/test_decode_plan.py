@@ -80,3 +80,23 @@ def test_random_and_extreme_decode_plans(checker, sms):
     cases.append((16, 2, [1], [1 << 25]))                                 # the longest decode row
     for case, line in zip(cases, _run(checker, cases, sms)):
         assert line.startswith("ok"), f"{case[:2]} {len(case[2])} rows: {line}"
+
+
+def test_cluster_plans_only_where_the_merge_bounds_the_step(checker):
+    """With the co-resident cluster capacity of a GB300 (36 clusters of 4 of
+    the decode kernel), the plan puts the splits of a Qwen2.5-3B step of one
+    or two decode rows into clusters of 4 (the split merge reads a quarter of
+    the partials) and keeps plain CTAs where clusters would leave SMs idle or
+    unbalance the splits (4 and 8 rows, 16 Llama rows), and for any step with
+    prefill rows (a mixed launch has no clusters)."""
+    q3, l8 = wl.QWEN25_3B, wl.LLAMA31_8B
+    cases = [("qwen 1 row", q3, [1], [25000], 4),
+             ("qwen 2 rows", q3, [1, 1], [25000, 25020], 4),
+             ("qwen 4 rows", q3, [1] * 4, [25000, 25010, 25020, 25030], 1),
+             ("qwen 8 rows", q3, [1] * 8, [25000 + 4 * i for i in range(8)], 1),
+             ("llama 16 rows", l8, [1] * 16, [30000 + 4 * i for i in range(16)], 1),
+             ("qwen 1 row beside a chunk", q3, [1, 512], [25000, 2048], 1)]
+    lines = _run(checker, [(g.n_q_heads, g.n_kv_heads, q, c) for _, g, q, c, _ in cases])
+    for (name, _, _, _, want), line in zip(cases, lines):
+        assert line.startswith("ok"), f"{name}: {line}"
+        assert int(line.split()[3]) == want, f"{name}: {line}"
