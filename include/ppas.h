@@ -289,7 +289,8 @@ ppas_status ppas_gateup_swiglu(const void *x, const void *w_packed, void *y, int
  *    magnitude (~4e-4 relative at 110k keys, ~5e-3 at 880k).
  *  - The first call on a device (with rows to run) does the library's
  *    one-time set-up for that device with it current: it looks up the
- *    array's device address, sets the kernels' shared-memory limits and
+ *    array's device address, sets the kernels' shared-memory limits,
+ *    queries how many decode clusters the device holds co-resident and
  *    creates the side stream and two events that steps too large for one
  *    launch use.  Make that first
  *    call before any stream capture and before a phase in which nothing may

@@ -17,8 +17,8 @@
 // call on each device looks the address up with cudaGetSymbolAddress while
 // that device is current, and later calls reuse it.  That first call also
 // does the library's other one-time set-up for the device (the kernels'
-// shared-memory limits, the side stream and events of mixed steps), so that
-// no later call creates anything.
+// shared-memory limits, the decode cluster capacity, the side stream and
+// events of mixed steps), so that no later call creates anything.
 #include <mutex>
 
 #include "ppas_internal.h"
@@ -55,7 +55,8 @@ extern "C" ppas_status ppas_attention_step_noalloc(const void *q, const void *k_
                                                    int32_t n_kv_heads, int32_t head_dim, float scale, void *out,
                                                    int32_t out_is_fp32, int32_t *d_err_flag, void *stream) {
     // the decode scratch this step needs must fit the fixed array (checked
-    // before any CUDA call); the prefill tiles' split partials are used when
+    // before any launch; on a device's first call the plan queries its
+    // cluster capacity); the prefill tiles' split partials are used when
     // they fit beside it, else the prefill tiles run unsplit
     const size_t need = ppas::workspace_min_size(n_seqs, h_q_lens, h_ctx_lens, n_q_heads, n_kv_heads);
     if (need > static_cast<size_t>(PPAS_NOALLOC_SCRATCH_BYTES)) return PPAS_ERR_CAPACITY;
