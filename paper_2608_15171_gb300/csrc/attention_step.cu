@@ -521,7 +521,7 @@ namespace {
 // iteration instead of once per layer (the stream-K search of a step like
 // MBT 2k takes ~70 us of host time).
 struct CachedPlan {
-    int32_t n = -1, hq = 0, hk = 0, sms = 0;
+    int32_t n = -1, hq = 0, hk = 0, sms = 0, clusters4 = 0;  // the device's SMs and cluster capacity
     size_t ws = 0;
     std::vector<int32_t> q, c;
     std::shared_ptr<const StepPlan> plan;
@@ -535,9 +535,10 @@ thread_local int t_plan_next = 0;
 std::shared_ptr<const StepPlan> plan_step_cached(int32_t n_seqs, const int32_t *q_lens, const int32_t *ctx_lens,
                                                  int32_t n_q_heads, int32_t n_kv_heads, size_t workspace_bytes) {
     const int32_t sms = plan_sms();
+    const int32_t clusters4 = decode_cluster_caps().ctas4;
     for (const CachedPlan &e : t_plans)
         if (e.plan && e.n == n_seqs && e.hq == n_q_heads && e.hk == n_kv_heads && e.sms == sms &&
-            e.ws == workspace_bytes && std::equal(q_lens, q_lens + n_seqs, e.q.begin()) &&
+            e.clusters4 == clusters4 && e.ws == workspace_bytes && std::equal(q_lens, q_lens + n_seqs, e.q.begin()) &&
             std::equal(ctx_lens, ctx_lens + n_seqs, e.c.begin()))
             return e.plan;
     auto sp = std::make_shared<const StepPlan>(
@@ -548,6 +549,7 @@ std::shared_ptr<const StepPlan> plan_step_cached(int32_t n_seqs, const int32_t *
     e.hq = n_q_heads;
     e.hk = n_kv_heads;
     e.sms = sms;
+    e.clusters4 = clusters4;
     e.ws = workspace_bytes;
     e.q.assign(q_lens, q_lens + n_seqs);
     e.c.assign(ctx_lens, ctx_lens + n_seqs);
